@@ -1,0 +1,142 @@
+"""PRECOG oracle: slow, sequential fp64 CPU reference of the hot path.
+
+TEST INFRASTRUCTURE ONLY. Only the test suite, ``__graft_entry__.smoke()`` and
+the CPU-baseline leg of ``bench.py`` may import this package. The product
+library never loads it and shares no code with it.
+
+The arithmetic lives in ``precog_oracle.c`` (plain C, double precision); this
+module compiles it with gcc and marshals numpy arrays into it.
+
+* :func:`scan` -- the selective-SSM rollout of Eq. 1 / Appendix A over every
+  chunk of one layer, with final-state capture (Sec. 4.2) and optional
+  readout ``y_t = C(h_t)``.
+* :func:`retrieve` -- exact top-1 dot-product retrieval (Sec. 4.2), lowest row
+  on ties, NaN never wins.
+* :func:`rollout` -- one chunk convenience wrapper of :func:`scan`.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "precog_oracle.c")
+_BUILD_DIR = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD_DIR, "liboracle.so")
+
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile the C oracle into ``oracle/_build/liboracle.so`` (gcc, -O2,
+    no floating-point contraction, no fast-math) and return its path."""
+    with _lock:
+        if (not force and os.path.exists(_LIB_PATH)
+                and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+            return _LIB_PATH
+        os.makedirs(_BUILD_DIR, exist_ok=True)
+        tmp = _LIB_PATH + f".tmp{os.getpid()}"
+        cmd = ["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-fno-fast-math",
+               "-shared", "-fPIC", _SRC, "-o", tmp, "-lm"]
+        subprocess.run(cmd, check=True)
+        os.replace(tmp, _LIB_PATH)
+        return _LIB_PATH
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        build()
+        lib = ctypes.CDLL(_LIB_PATH)
+        p_i64 = ctypes.POINTER(ctypes.c_int64)
+        p_f64 = ctypes.POINTER(ctypes.c_double)
+        lib.oracle_scan.restype = ctypes.c_int
+        lib.oracle_scan.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, p_i64,
+                                    p_f64, p_f64, p_f64, p_f64, p_f64, p_f64, p_f64, p_f64]
+        lib.oracle_retrieve.restype = ctypes.c_int
+        lib.oracle_retrieve.argtypes = [ctypes.c_int64, ctypes.c_int64, p_f64, ctypes.c_int64,
+                                        p_f64, p_i64, p_f64]
+        _lib = lib
+    return _lib
+
+
+def _f64(a):
+    if a is None:
+        return None
+    return np.ascontiguousarray(np.asarray(a, dtype=np.float64))
+
+
+def _ptr(a, ctype):
+    if a is None:
+        return ctypes.POINTER(ctype)()
+    return a.ctypes.data_as(ctypes.POINTER(ctype))
+
+
+def scan(x, dt, A, B, offsets, C=None, h0=None, want_y=False):
+    """Scan one layer of chunks from ``h0`` (zero state when None).
+
+    Shapes: x, dt ``[T_tot, D]``; A ``[D, N]``; B, C ``[T_tot, N]``;
+    offsets ``[n_chunks + 1]`` int64 prefix sums; h0 ``[n_chunks, D, N]``.
+    Returns ``(states [n_chunks, D, N], y [T_tot, D] or None)`` in float64.
+    """
+    lib = _load()
+    x, dt, A, B = _f64(x), _f64(dt), _f64(A), _f64(B)
+    C = _f64(C) if want_y else None
+    h0 = _f64(h0)
+    offsets = np.ascontiguousarray(np.asarray(offsets, dtype=np.int64))
+    D, N = A.shape
+    n_chunks = offsets.shape[0] - 1
+    T_tot = x.shape[0]
+    if x.shape != (T_tot, D) or dt.shape != (T_tot, D) or B.shape != (T_tot, N):
+        raise ValueError("oracle.scan: inconsistent input shapes")
+    if want_y and (C is None or C.shape != (T_tot, N)):
+        raise ValueError("oracle.scan: y requested but C has the wrong shape")
+    if h0 is not None and h0.shape != (n_chunks, D, N):
+        raise ValueError("oracle.scan: h0 must be [n_chunks, D, N]")
+    if n_chunks > 0 and (offsets[0] < 0 or offsets[-1] > T_tot):
+        raise ValueError("oracle.scan: offsets out of range")
+    states = np.zeros((n_chunks, D, N), dtype=np.float64)
+    y = np.zeros((T_tot, D), dtype=np.float64) if want_y else None
+    p64, pi = ctypes.c_double, ctypes.c_int64
+    rc = lib.oracle_scan(D, N, n_chunks, _ptr(offsets, pi), _ptr(x, p64), _ptr(dt, p64),
+                         _ptr(A, p64), _ptr(B, p64), _ptr(C, p64), _ptr(h0, p64),
+                         _ptr(states, p64), _ptr(y, p64))
+    if rc != 0:
+        raise ValueError(f"oracle_scan rejected its arguments (rc={rc})")
+    return states, y
+
+
+def rollout(x, dt, A, B, C=None, h0=None, want_y=False):
+    """S(h0, x_{1:T}) of Appendix A for one chunk: returns ``(h_T [D, N], y [T, D])``."""
+    x = _f64(x)
+    T = x.shape[0]
+    D, N = np.asarray(A).shape
+    h0b = None if h0 is None else _f64(h0).reshape(1, D, N)
+    states, y = scan(x, dt, A, B, np.array([0, T], dtype=np.int64), C=C, h0=h0b, want_y=want_y)
+    return states[0], y
+
+
+def retrieve(index, queries):
+    """Exact top-1 by dot product; returns ``(best_idx int64 [Q], best_score float64 [Q])``."""
+    lib = _load()
+    index = _f64(index)
+    queries = _f64(queries)
+    if queries.ndim == 1:
+        queries = queries.reshape(1, -1)
+    M, dim = index.shape
+    Q = queries.shape[0]
+    if queries.shape[1] != dim:
+        raise ValueError("oracle.retrieve: query dim mismatch")
+    best_idx = np.empty(Q, dtype=np.int64)
+    best_score = np.empty(Q, dtype=np.float64)
+    rc = lib.oracle_retrieve(M, dim, _ptr(index, ctypes.c_double), Q,
+                             _ptr(queries, ctypes.c_double),
+                             _ptr(best_idx, ctypes.c_int64), _ptr(best_score, ctypes.c_double))
+    if rc != 0:
+        raise ValueError(f"oracle_retrieve rejected its arguments (rc={rc})")
+    return best_idx, best_score

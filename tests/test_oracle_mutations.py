@@ -1,0 +1,70 @@
+"""The oracle's pins have teeth: plant a plausible mistake in a copy of the C oracle,
+compile it on the CPU, and check that at least one pin test fails against it."""
+import ctypes
+import os
+import subprocess
+
+import pytest
+
+import oracle
+from tests import test_oracle_pins as pins
+
+SRC = os.path.join(os.path.dirname(oracle.__file__), "precog_oracle.c")
+
+MUTATIONS = {
+    "dropped_beta": ("h[n] = h[n] * alpha + beta;", "h[n] = h[n] * alpha;"),
+    "exponent_sign": ("exp(dt_td * A[d * N + n])", "exp(-dt_td * A[d * N + n])"),
+    "transposed_A": ("exp(dt_td * A[d * N + n])", "exp(dt_td * A[n * D + d])"),
+    "B_by_channel": ("B[t * N + n] * x_td", "B[t * N + (d % N)] * x_td"),
+    "beta_without_dt": ("B[t * N + n] * x_td * dt_td", "B[t * N + n] * x_td"),
+    "readout_wrong_state": ("C[t * N + n] * h[n]", "C[t * N + n] * h[(n + 1) % N]"),
+    "chunk_end_off_by_one": ("t < offsets[c + 1]; ++t", "t + 1 < offsets[c + 1]; ++t"),
+    "ties_go_high": ("if (s > best)", "if (s >= best)"),
+}
+
+PIN_TESTS = [
+    lambda: pins.test_theorem1_precog_equals_in_context(37, 11),
+    pins.test_proposition_outputs_depend_on_context_only_through_state,
+    pins.test_constant_gates_geometric_series,
+    pins.test_A_zero_is_cumulative_sum_exact,
+    pins.test_dyadic_gates_hand_expanded,
+    pins.test_readout_uses_updated_state,
+    lambda: pins.test_unroll_closed_form_and_linearity(5),
+    pins.test_channel_isolation_and_state_index,
+    pins.test_chunk_boundaries_and_empty_chunks,
+    pins.test_stability_bound,
+    pins.test_retrieve_matches_numpy_argmax_first_occurrence,
+    pins.test_retrieve_ties_nan_and_empty,
+    pins.test_retrieve_planted_tiny_workload,
+]
+
+
+def _compile(src_text, out_dir, name):
+    c_path = os.path.join(out_dir, f"{name}.c")
+    so_path = os.path.join(out_dir, f"{name}.so")
+    with open(c_path, "w") as f:
+        f.write(src_text)
+    subprocess.run(["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-shared", "-fPIC",
+                    c_path, "-o", so_path, "-lm"], check=True)
+    return so_path
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_planted_mistake_is_caught(name, tmp_path, monkeypatch):
+    src = open(SRC).read()
+    old, new = MUTATIONS[name]
+    assert old in src, f"mutation anchor for {name} not found in the oracle source"
+    so_path = _compile(src.replace(old, new), str(tmp_path), name)
+    real = oracle._load()
+    mutant = ctypes.CDLL(so_path)
+    for fn in ("oracle_scan", "oracle_retrieve"):
+        getattr(mutant, fn).restype = getattr(real, fn).restype
+        getattr(mutant, fn).argtypes = getattr(real, fn).argtypes
+    monkeypatch.setattr(oracle, "_lib", mutant)
+    failures = 0
+    for pin in PIN_TESTS:
+        try:
+            pin()
+        except AssertionError:
+            failures += 1
+    assert failures > 0, f"no pin caught the planted mistake '{name}'"
