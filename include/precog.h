@@ -1,0 +1,198 @@
+/*
+ * precog.h -- C ABI of the PRECOG hot path on one GB300 GPU (sm_103a).
+ *
+ * PRECOG (Sec. 4 of "Structured Memory for Edge Language Models: Persistent
+ * Context and Corpus Retrieval via O(1) SSM State Injection") pre-encodes
+ * corpus chunks into the final hidden state of a selective SSM (offline
+ * indexing, Sec. 4.2), retrieves the best-matching chunk for a query by
+ * embedding similarity, injects that chunk's state as the recurrence's initial
+ * condition (Eq. 2) and prefills only the query tokens from it. Theorem 1
+ * guarantees this equals scanning [chunk; query] from the zero state.
+ *
+ * Conventions shared by every call
+ *   - All data pointers are DEVICE pointers owned by the caller; the library
+ *     allocates nothing. Each must be 16-byte aligned.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream). Every call only enqueues work on it and returns; results are
+ *     ready when the stream reaches that point.
+ *   - Argument errors are detected on the host before anything is enqueued;
+ *     the call then returns PRECOG_ERR_INVALID_ARG or PRECOG_ERR_UNSUPPORTED and
+ *     leaves every output untouched. precog_last_error() describes the cause.
+ *   - Errors that only the device can see (a bad chunk offset, an out-of-range
+ *     bank row, a pipeline wait that gave up) are recorded in a device status
+ *     word instead of faulting; precog_device_status() reports and clears it.
+ *   - Floating point: the recurrence and every accumulation run in fp32.
+ *   - No call raises a C++ exception or aborts across this boundary.
+ */
+#ifndef PRECOG_H_
+#define PRECOG_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define PRECOG_ABI_VERSION 1
+
+typedef enum precog_status {
+    PRECOG_OK = 0,
+    PRECOG_ERR_INVALID_ARG = 1,  /* a pointer, size or layout argument is invalid */
+    PRECOG_ERR_UNSUPPORTED = 2,  /* valid, but outside what the kernels implement */
+    PRECOG_ERR_CUDA = 3,         /* a CUDA runtime call or a launch failed */
+    PRECOG_ERR_TIMEOUT = 4,      /* a bounded device-side wait gave up */
+    PRECOG_ERR_DEVICE = 5        /* the device flagged bad offsets or bank rows */
+} precog_status;
+
+typedef enum precog_dtype {
+    PRECOG_F32 = 0,
+    PRECOG_BF16 = 1,
+    PRECOG_F16 = 2
+} precog_dtype;
+
+/* Device status bits reported by precog_device_status(). */
+#define PRECOG_DEV_BAD_OFFSETS 0x1u  /* offsets not non-decreasing or beyond T_tot */
+#define PRECOG_DEV_BAD_INDEX 0x2u    /* a bank row index outside [-1, bank_entries) */
+#define PRECOG_DEV_TIMEOUT 0x4u      /* an mbarrier wait hit its iteration limit */
+
+/*
+ * Inputs of the selective-SSM scan for L layers (Sec. 3, Eq. 1).
+ *
+ * Per layer l, channel d, state index n and token row t:
+ *   alpha = exp(dt[t,d] * A[d,n])     (A < 0: the stable reading of Eq. 1)
+ *   h[d,n] <- alpha * h[d,n] + B[t,n] * x[t,d] * dt[t,d]
+ *   y[t,d]  = sum_n C[t,n] * h[d,n]   (readout of the updated state)
+ * dt is per (token, channel) and B, C per (token, state index), shared across
+ * channels: the input-dependent timescale and projections of a selective SSM
+ * ("dt and B are functions of the current token only", Sec. 3).
+ *
+ * Layout (row-major, element strides):
+ *   x, dt : layer l at  x + l*layer_stride_xd, each block [T_tot][D]
+ *   B, C  : layer l at  B + l*layer_stride_bc, each block [T_tot][N]
+ *   A     : [L][D][N] fp32, always dense
+ * x, dt, B, C share `in_dtype` (PRECOG_F32 or PRECOG_BF16). C may be NULL
+ * when no readout is requested. Strides are in elements and must keep every
+ * layer block 16-byte aligned; they may be 0 when n_layers == 1.
+ * Requirements: N == 16; D >= 1 with D*sizeof(in_dtype) a multiple of 16.
+ * x, dt and B (and C) may be NULL only when there are no token rows.
+ * When A[d,n] == (n+1)*A[d,0] holds exactly for every n of a channel group,
+ * the kernel derives alpha_n as a power of one exponential (the same value
+ * up to fp32 rounding); otherwise it takes one exponential per (d, n).
+ */
+typedef struct precog_scan_inputs {
+    int32_t n_layers;
+    int32_t D;
+    int32_t N;
+    int32_t in_dtype;          /* precog_dtype */
+    const void *x;
+    const void *dt;
+    const void *B;
+    const void *C;
+    const float *A;
+    int64_t layer_stride_xd;
+    int64_t layer_stride_bc;
+} precog_scan_inputs;
+
+/*
+ * precog_encode_chunks -- offline indexing (Sec. 4.2): scan every chunk of a
+ * ragged batch from the zero state (Appendix B.1) through L layers and capture
+ * each chunk's final per-layer state h(c) = S(0, c) (Theorem 1 notation).
+ *
+ *   in          scan inputs, L = in->n_layers layers, T_tot token rows each
+ *   d_offsets   device int64 [n_chunks+1]: chunk c owns rows
+ *               d_offsets[c] .. d_offsets[c+1]-1 of every layer; must be
+ *               non-decreasing with d_offsets[n_chunks] <= T_tot (checked on
+ *               the device: a bad chunk is skipped and flags
+ *               PRECOG_DEV_BAD_OFFSETS). A zero-length chunk captures zeros.
+ *   states_out  device [n_chunks][L_total][D][N] in state_dtype (F32 or BF16,
+ *               rounded to nearest even once, at capture); the call writes
+ *               layers layer0 .. layer0+L-1 and nothing else. May be NULL
+ *               when y_out is given.
+ *   y_out       device [L][T_tot][D] in y_dtype (F32 or BF16): readout after
+ *               every token (used to check Theorem 1), or NULL for capture
+ *               only. Rows outside every chunk are left untouched.
+ * Returns PRECOG_OK once the work is enqueued.
+ */
+precog_status precog_encode_chunks(const precog_scan_inputs *in, const int64_t *d_offsets,
+                                   int64_t n_chunks, int64_t T_tot, void *states_out,
+                                   int32_t state_dtype, int32_t layer0, int32_t L_total,
+                                   void *y_out, int32_t y_dtype, void *stream);
+
+/*
+ * precog_retrieve -- query-time retrieval (Sec. 4.2): for every query q the
+ * row i* of the key index with the highest dot product <query_q, key_i>
+ * (unit-norm keys and queries make this the cosine similarity of the paper).
+ * Exact top-1, not an approximate index. Scores accumulate in fp32 from the
+ * stored values; ties go to the lowest row; a NaN score never wins; if no row
+ * has a comparable score the result is index -1 and score NaN.
+ *
+ *   index          device [M][dim] keys in index_dtype (F16, BF16 or F32)
+ *   queries        device [n_queries][dim], same dtype as the index
+ *   d_best_idx     device int64 [n_queries] (written)
+ *   d_best_score   device fp32 [n_queries] (written), or NULL
+ *   workspace      device scratch of at least
+ *                  precog_retrieve_workspace_size(M, dim, n_queries) bytes;
+ *                  contents on entry are ignored and clobbered
+ * Requirements: 0 <= M < 2^31 - 1; dim >= 1 with dim*sizeof(dtype) a
+ * multiple of 16; n_queries >= 0.
+ */
+precog_status precog_retrieve(const void *index, int32_t index_dtype, int64_t M, int32_t dim,
+                              const void *queries, int32_t n_queries, int64_t *d_best_idx,
+                              float *d_best_score, void *workspace, size_t workspace_bytes,
+                              void *stream);
+
+/* Bytes of device workspace precog_retrieve needs for these sizes. */
+size_t precog_retrieve_workspace_size(int64_t M, int32_t dim, int32_t n_queries);
+
+/*
+ * precog_prefill_from_state -- state injection and query prefill (Sec. 4.2,
+ * Eq. 2): for every query q and layer l, h_init[l] <- bank[row_q][layer0+l],
+ * then scan the query's T_q tokens from h_init, producing y_t for every query
+ * token and the updated state. By Theorem 1 this equals scanning
+ * [chunk; query] from the zero state.
+ *
+ *   in           scan inputs with T_tot = n_queries*T_q rows per layer: query
+ *                q owns rows q*T_q .. q*T_q+T_q-1; C is required when y_out
+ *                is given
+ *   bank         device [bank_entries][L_bank][D][N] in bank_dtype (F32/BF16)
+ *   d_idx        device int64 [n_queries]: bank row injected for query q
+ *                (e.g. precog_retrieve's d_best_idx, read on the device with
+ *                no host round trip). -1 injects the zero state (no context).
+ *                Other rows outside [0, bank_entries) also inject zeros and
+ *                flag PRECOG_DEV_BAD_INDEX. NULL means row q for query q.
+ *   layer0       first bank layer used; layers layer0 .. layer0+L-1 must be
+ *                < L_bank
+ *   y_out        device [L][n_queries*T_q][D] in y_dtype, or NULL
+ *   state_out    device [n_queries][L_bank][D][N] in state_dtype (layers
+ *                layer0 .. layer0+L-1 written), or NULL
+ */
+precog_status precog_prefill_from_state(const precog_scan_inputs *in, int32_t n_queries,
+                                        int32_t T_q, const void *bank, int32_t bank_dtype,
+                                        int64_t bank_entries, int32_t L_bank, int32_t layer0,
+                                        const int64_t *d_idx, void *y_out, int32_t y_dtype,
+                                        void *state_out, int32_t state_dtype, void *stream);
+
+/*
+ * precog_device_status -- synchronise `stream`, then report and clear the
+ * device status word shared by all calls on this device. *bits_out receives
+ * the PRECOG_DEV_* bits seen since the last clear. Returns PRECOG_OK when no
+ * bit was set, PRECOG_ERR_TIMEOUT when PRECOG_DEV_TIMEOUT was set, otherwise
+ * PRECOG_ERR_DEVICE; PRECOG_ERR_CUDA if the synchronisation itself failed.
+ */
+precog_status precog_device_status(void *stream, uint32_t *bits_out);
+
+/* Human-readable name of a status code (static storage). */
+const char *precog_status_string(int32_t status);
+
+/* Detail of the last error returned on the calling thread ("" if none). */
+const char *precog_last_error(void);
+
+/* PRECOG_ABI_VERSION of the loaded library. */
+int32_t precog_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PRECOG_H_ */

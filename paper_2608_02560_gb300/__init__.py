@@ -1,0 +1,191 @@
+"""PRECOG hot path on GB300: Python binding of the C-ABI library ``libprecog.so``.
+
+Thin ctypes marshalling only: every step of the path (scan with state capture,
+top-1 retrieval, state injection and query prefill) runs in the library's CUDA
+kernels. PyTorch tensors are accepted for device memory and the current CUDA
+stream; nothing here computes. If the library is missing the import fails
+loudly: there is no CPU fallback.
+
+Functions carry the C names:
+
+* :func:`precog_encode_chunks`    -- offline indexing (Sec. 4.2)
+* :func:`precog_retrieve`         -- exact top-1 retrieval (Sec. 4.2)
+* :func:`precog_prefill_from_state` -- injection (Eq. 2) + query prefill
+* :func:`precog_device_status`    -- device-side status word
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libprecog.so")
+
+PRECOG_F32, PRECOG_BF16, PRECOG_F16 = 0, 1, 2
+PRECOG_OK = 0
+PRECOG_DEV_BAD_OFFSETS, PRECOG_DEV_BAD_INDEX, PRECOG_DEV_TIMEOUT = 0x1, 0x2, 0x4
+STATUS_NAMES = {0: "PRECOG_OK", 1: "PRECOG_ERR_INVALID_ARG", 2: "PRECOG_ERR_UNSUPPORTED",
+                3: "PRECOG_ERR_CUDA", 4: "PRECOG_ERR_TIMEOUT", 5: "PRECOG_ERR_DEVICE"}
+
+
+class PrecogError(RuntimeError):
+    def __init__(self, status: int, detail: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {detail}")
+        self.status = status
+        self.detail = detail
+
+
+class ScanInputs(ctypes.Structure):
+    """Mirror of ``precog_scan_inputs`` (include/precog.h)."""
+    _fields_ = [("n_layers", ctypes.c_int32), ("D", ctypes.c_int32), ("N", ctypes.c_int32),
+                ("in_dtype", ctypes.c_int32), ("x", ctypes.c_void_p), ("dt", ctypes.c_void_p),
+                ("B", ctypes.c_void_p), ("C", ctypes.c_void_p), ("A", ctypes.c_void_p),
+                ("layer_stride_xd", ctypes.c_int64), ("layer_stride_bc", ctypes.c_int64)]
+
+
+_lib = None
+
+
+def load_library(path: str = LIB_PATH):
+    """Load ``libprecog.so`` (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise ImportError(f"libprecog.so not found at {path}; build it with "
+                          "`python -m paper_2608_02560_gb300.build`")
+    lib = ctypes.CDLL(path)
+    i32, i64, vp, sz = ctypes.c_int32, ctypes.c_int64, ctypes.c_void_p, ctypes.c_size_t
+    lib.precog_encode_chunks.restype = i32
+    lib.precog_encode_chunks.argtypes = [ctypes.POINTER(ScanInputs), vp, i64, i64, vp, i32, i32,
+                                         i32, vp, i32, vp]
+    lib.precog_retrieve.restype = i32
+    lib.precog_retrieve.argtypes = [vp, i32, i64, i32, vp, i32, vp, vp, vp, sz, vp]
+    lib.precog_retrieve_workspace_size.restype = sz
+    lib.precog_retrieve_workspace_size.argtypes = [i64, i32, i32]
+    lib.precog_prefill_from_state.restype = i32
+    lib.precog_prefill_from_state.argtypes = [ctypes.POINTER(ScanInputs), i32, i32, vp, i32, i64,
+                                              i32, i32, vp, vp, i32, vp, i32, vp]
+    lib.precog_device_status.restype = i32
+    lib.precog_device_status.argtypes = [vp, ctypes.POINTER(ctypes.c_uint32)]
+    lib.precog_status_string.restype = ctypes.c_char_p
+    lib.precog_status_string.argtypes = [i32]
+    lib.precog_last_error.restype = ctypes.c_char_p
+    lib.precog_last_error.argtypes = []
+    lib.precog_abi_version.restype = i32
+    lib.precog_abi_version.argtypes = []
+    _lib = lib
+    return lib
+
+
+def _check(status: int):
+    if status != PRECOG_OK:
+        raise PrecogError(status, load_library().precog_last_error().decode())
+
+
+# ------------------------------------------------------------------------------- marshalling
+
+
+def _dtype_code(t) -> int:
+    import torch
+    m = {torch.float32: PRECOG_F32, torch.bfloat16: PRECOG_BF16, torch.float16: PRECOG_F16}
+    if t.dtype not in m:
+        raise TypeError(f"unsupported dtype {t.dtype}")
+    return m[t.dtype]
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("tensors passed to libprecog must live on the GPU")
+    if not t.is_contiguous():
+        raise ValueError("tensors passed to libprecog must be contiguous")
+    return t.data_ptr()
+
+
+def _stream(stream):
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def scan_inputs(x, dt, B, A, C=None) -> ScanInputs:
+    """Describe x, dt ``[L, T, D]`` (or ``[T, D]``), B, C ``[L, T, N]``, A ``[L, D, N]``."""
+    if x.dim() == 2:
+        x, dt, B = x.unsqueeze(0), dt.unsqueeze(0), B.unsqueeze(0)
+        C = None if C is None else C.unsqueeze(0)
+    if A.dim() == 2:
+        A = A.unsqueeze(0)
+    L, T, D = x.shape
+    N = B.shape[-1]
+    if dt.shape != x.shape or B.shape != (L, T, N) or (C is not None and C.shape != B.shape):
+        raise ValueError("x/dt/B/C shapes disagree")
+    import torch
+    if A.shape != (L, D, N) or A.dtype != torch.float32:
+        raise ValueError("A must be float32 [L, D, N]")
+    s = ScanInputs()
+    s.n_layers, s.D, s.N = L, D, N
+    s.in_dtype = _dtype_code(x)
+    s.x, s.dt, s.B, s.C, s.A = _ptr(x), _ptr(dt), _ptr(B), _ptr(C), _ptr(A)
+    s.layer_stride_xd = T * D
+    s.layer_stride_bc = T * N
+    return s
+
+
+# ------------------------------------------------------------------------------- the C calls
+
+
+def precog_encode_chunks(inputs: ScanInputs, offsets, T_tot: int, states_out=None,
+                         layer0: int = 0, L_total: int | None = None, y_out=None, stream=None):
+    """Scan every chunk (rows ``offsets[c]..offsets[c+1]``) from zero; capture final states
+    into ``states_out [n_chunks, L_total, D, N]`` and/or readouts into ``y_out [L, T_tot, D]``."""
+    lib = load_library()
+    n_chunks = offsets.numel() - 1
+    if L_total is None:
+        L_total = inputs.n_layers
+    _check(lib.precog_encode_chunks(
+        ctypes.byref(inputs), _ptr(offsets), n_chunks, T_tot, _ptr(states_out),
+        _dtype_code(states_out) if states_out is not None else PRECOG_F32, layer0, L_total,
+        _ptr(y_out), _dtype_code(y_out) if y_out is not None else PRECOG_F32, _stream(stream)))
+
+
+def precog_retrieve_workspace_size(M: int, dim: int, n_queries: int) -> int:
+    return int(load_library().precog_retrieve_workspace_size(M, dim, n_queries))
+
+
+def precog_retrieve(index, queries, best_idx, best_score=None, workspace=None, stream=None):
+    """Exact top-1 of ``queries [Q, dim]`` against ``index [M, dim]`` into int64 ``best_idx``
+    and fp32 ``best_score``. ``workspace`` is allocated with torch when not given."""
+    import torch
+    lib = load_library()
+    M, dim = index.shape
+    Q = queries.shape[0]
+    need = precog_retrieve_workspace_size(M, dim, Q)
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=index.device)
+    _check(lib.precog_retrieve(
+        _ptr(index), _dtype_code(index), M, dim, _ptr(queries), Q, _ptr(best_idx),
+        _ptr(best_score), _ptr(workspace), workspace.numel() * workspace.element_size(),
+        _stream(stream)))
+
+
+def precog_prefill_from_state(inputs: ScanInputs, n_queries: int, T_q: int, bank, idx=None,
+                              layer0: int = 0, y_out=None, state_out=None, stream=None):
+    """Inject ``bank[idx[q]]`` (``[entries, L_bank, D, N]``) and scan each query's T_q tokens."""
+    lib = load_library()
+    entries, L_bank = bank.shape[0], bank.shape[1]
+    _check(lib.precog_prefill_from_state(
+        ctypes.byref(inputs), n_queries, T_q, _ptr(bank), _dtype_code(bank), entries, L_bank,
+        layer0, _ptr(idx), _ptr(y_out), _dtype_code(y_out) if y_out is not None else PRECOG_F32,
+        _ptr(state_out), _dtype_code(state_out) if state_out is not None else PRECOG_F32,
+        _stream(stream)))
+
+
+def precog_device_status(stream=None):
+    """Synchronise the stream and return (status, bits) of the device status word (cleared)."""
+    lib = load_library()
+    bits = ctypes.c_uint32(0)
+    st = lib.precog_device_status(_stream(stream), ctypes.byref(bits))
+    return st, bits.value

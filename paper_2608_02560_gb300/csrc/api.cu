@@ -1,0 +1,252 @@
+// C ABI of the PRECOG hot path: argument validation, dispatch to the
+// kernels, status codes. Nothing here allocates device memory.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+
+#include "../../include/precog.h"
+#include "internal.h"
+
+namespace {
+
+thread_local char g_last_error[512] = "";
+
+precog_status fail(precog_status s, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_last_error, sizeof(g_last_error), fmt, ap);
+    va_end(ap);
+    return s;
+}
+
+precog_status ok() {
+    g_last_error[0] = '\0';
+    return PRECOG_OK;
+}
+
+precog_status cuda_fail(cudaError_t e, const char *what) {
+    return fail(PRECOG_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int dtype_size(int32_t dt) {
+    switch (dt) {
+        case PRECOG_F32: return 4;
+        case PRECOG_BF16: return 2;
+        case PRECOG_F16: return 2;
+        default: return 0;
+    }
+}
+
+bool state_dtype_ok(int32_t dt) { return dt == PRECOG_F32 || dt == PRECOG_BF16; }
+
+// Checks shared by encode and prefill. rows = T_tot per layer.
+precog_status check_scan_inputs(const precog_scan_inputs *in, int64_t rows, bool need_C) {
+    if (in == nullptr) return fail(PRECOG_ERR_INVALID_ARG, "scan inputs pointer is NULL");
+    if (in->n_layers < 1) return fail(PRECOG_ERR_INVALID_ARG, "n_layers must be >= 1");
+    if (in->N != 16) return fail(PRECOG_ERR_UNSUPPORTED, "N=%d: only N=16 is implemented", in->N);
+    if (in->D < 1) return fail(PRECOG_ERR_INVALID_ARG, "D must be >= 1");
+    if (in->in_dtype != PRECOG_F32 && in->in_dtype != PRECOG_BF16)
+        return fail(PRECOG_ERR_UNSUPPORTED, "in_dtype must be PRECOG_F32 or PRECOG_BF16");
+    const int sz = dtype_size(in->in_dtype);
+    if ((static_cast<int64_t>(in->D) * sz) % 16 != 0)
+        return fail(PRECOG_ERR_UNSUPPORTED, "D*sizeof(in_dtype) must be a multiple of 16");
+    if (in->A == nullptr) return fail(PRECOG_ERR_INVALID_ARG, "A must be non-NULL");
+    if (rows > 0 && (in->x == nullptr || in->dt == nullptr || in->B == nullptr))
+        return fail(PRECOG_ERR_INVALID_ARG, "x, dt and B must be non-NULL");
+    if (rows > 0 && need_C && in->C == nullptr)
+        return fail(PRECOG_ERR_INVALID_ARG, "C is required when y_out is given");
+    if (!aligned16(in->x) || !aligned16(in->dt) || !aligned16(in->B) || !aligned16(in->A) ||
+        (in->C && !aligned16(in->C)))
+        return fail(PRECOG_ERR_INVALID_ARG, "input pointers must be 16-byte aligned");
+    if (in->n_layers > 1) {
+        if (in->layer_stride_xd < rows * in->D || in->layer_stride_bc < rows * in->N)
+            return fail(PRECOG_ERR_INVALID_ARG, "layer strides smaller than one layer block");
+        if ((in->layer_stride_xd * sz) % 16 != 0 || (in->layer_stride_bc * sz) % 16 != 0)
+            return fail(PRECOG_ERR_INVALID_ARG, "layer strides must keep 16-byte alignment");
+    }
+    return PRECOG_OK;
+}
+
+precog::ScanParams base_params(const precog_scan_inputs *in, int64_t rows) {
+    precog::ScanParams p;
+    std::memset(&p, 0, sizeof(p));
+    p.x = in->x;
+    p.dt = in->dt;
+    p.B = in->B;
+    p.C = in->C;
+    p.A = in->A;
+    p.ls_xd = in->n_layers > 1 ? in->layer_stride_xd : 0;
+    p.ls_bc = in->n_layers > 1 ? in->layer_stride_bc : 0;
+    p.n_layers = in->n_layers;
+    p.D = in->D;
+    p.N = in->N;
+    p.in_dtype = in->in_dtype;
+    p.T_tot = rows;
+    return p;
+}
+
+}  // namespace
+
+extern "C" {
+
+precog_status precog_encode_chunks(const precog_scan_inputs *in, const int64_t *d_offsets,
+                                   int64_t n_chunks, int64_t T_tot, void *states_out,
+                                   int32_t state_dtype, int32_t layer0, int32_t L_total,
+                                   void *y_out, int32_t y_dtype, void *stream) {
+    if (T_tot < 0) return fail(PRECOG_ERR_INVALID_ARG, "T_tot must be >= 0");
+    precog_status s = check_scan_inputs(in, T_tot, y_out != nullptr);
+    if (s != PRECOG_OK) return s;
+    if (n_chunks < 0) return fail(PRECOG_ERR_INVALID_ARG, "n_chunks must be >= 0");
+    if (d_offsets == nullptr) return fail(PRECOG_ERR_INVALID_ARG, "d_offsets is NULL");
+    if (states_out == nullptr && y_out == nullptr)
+        return fail(PRECOG_ERR_INVALID_ARG, "states_out and y_out are both NULL: nothing to do");
+    if (states_out) {
+        if (!state_dtype_ok(state_dtype))
+            return fail(PRECOG_ERR_UNSUPPORTED, "state_dtype must be PRECOG_F32 or PRECOG_BF16");
+        if (!aligned16(states_out)) return fail(PRECOG_ERR_INVALID_ARG, "states_out not 16-byte aligned");
+        if (layer0 < 0 || L_total < 1 || layer0 + in->n_layers > L_total)
+            return fail(PRECOG_ERR_INVALID_ARG, "layers [layer0, layer0+n_layers) exceed L_total");
+    }
+    if (y_out) {
+        if (!state_dtype_ok(y_dtype))
+            return fail(PRECOG_ERR_UNSUPPORTED, "y_dtype must be PRECOG_F32 or PRECOG_BF16");
+        if (!aligned16(y_out)) return fail(PRECOG_ERR_INVALID_ARG, "y_out not 16-byte aligned");
+    }
+    if (n_chunks == 0) return ok();
+    precog::ScanParams p = base_params(in, T_tot);
+    p.offsets = d_offsets;
+    p.n_chunks = n_chunks;
+    p.states = states_out;
+    p.state_dtype = state_dtype;
+    p.L_out = L_total;
+    p.layer0 = states_out ? layer0 : 0;
+    p.y = y_out;
+    p.y_dtype = y_dtype;
+    cudaError_t e = precog::launch_scan(p, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "scan launch");
+    return ok();
+}
+
+precog_status precog_prefill_from_state(const precog_scan_inputs *in, int32_t n_queries,
+                                        int32_t T_q, const void *bank, int32_t bank_dtype,
+                                        int64_t bank_entries, int32_t L_bank, int32_t layer0,
+                                        const int64_t *d_idx, void *y_out, int32_t y_dtype,
+                                        void *state_out, int32_t state_dtype, void *stream) {
+    if (n_queries < 0 || T_q < 0) return fail(PRECOG_ERR_INVALID_ARG, "n_queries and T_q must be >= 0");
+    const int64_t rows = static_cast<int64_t>(n_queries) * T_q;
+    precog_status s = check_scan_inputs(in, rows, y_out != nullptr);
+    if (s != PRECOG_OK) return s;
+    if (bank == nullptr) return fail(PRECOG_ERR_INVALID_ARG, "bank is NULL");
+    if (!state_dtype_ok(bank_dtype))
+        return fail(PRECOG_ERR_UNSUPPORTED, "bank_dtype must be PRECOG_F32 or PRECOG_BF16");
+    if (!aligned16(bank)) return fail(PRECOG_ERR_INVALID_ARG, "bank not 16-byte aligned");
+    if (bank_entries < 0) return fail(PRECOG_ERR_INVALID_ARG, "bank_entries must be >= 0");
+    if (L_bank < 1 || layer0 < 0 || layer0 + in->n_layers > L_bank)
+        return fail(PRECOG_ERR_INVALID_ARG, "layers [layer0, layer0+n_layers) exceed L_bank");
+    if (d_idx == nullptr && bank_entries < n_queries)
+        return fail(PRECOG_ERR_INVALID_ARG, "d_idx is NULL but bank has fewer rows than queries");
+    if (y_out == nullptr && state_out == nullptr)
+        return fail(PRECOG_ERR_INVALID_ARG, "y_out and state_out are both NULL: nothing to do");
+    if (y_out && (!state_dtype_ok(y_dtype) || !aligned16(y_out)))
+        return fail(PRECOG_ERR_INVALID_ARG, "y_out must be 16-byte aligned F32 or BF16");
+    if (state_out && (!state_dtype_ok(state_dtype) || !aligned16(state_out)))
+        return fail(PRECOG_ERR_INVALID_ARG, "state_out must be 16-byte aligned F32 or BF16");
+    if (n_queries == 0) return ok();
+    precog::ScanParams p = base_params(in, rows);
+    p.n_chunks = n_queries;
+    p.use_fixed = 1;
+    p.fixed_len = T_q;
+    p.bank = bank;
+    p.bank_dtype = bank_dtype;
+    p.bank_entries = bank_entries;
+    p.idx = d_idx;
+    p.L_bank = L_bank;
+    p.states = state_out;
+    p.state_dtype = state_dtype;
+    p.L_out = L_bank;
+    p.layer0 = layer0;
+    p.y = y_out;
+    p.y_dtype = y_dtype;
+    cudaError_t e = precog::launch_scan(p, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "prefill launch");
+    return ok();
+}
+
+size_t precog_retrieve_workspace_size(int64_t M, int32_t dim, int32_t n_queries) {
+    if (M < 0 || dim < 1 || n_queries < 0) return 0;
+    return precog::retrieve_workspace_size(M, dim, n_queries);
+}
+
+precog_status precog_retrieve(const void *index, int32_t index_dtype, int64_t M, int32_t dim,
+                              const void *queries, int32_t n_queries, int64_t *d_best_idx,
+                              float *d_best_score, void *workspace, size_t workspace_bytes,
+                              void *stream) {
+    const int sz = dtype_size(index_dtype);
+    if (sz == 0) return fail(PRECOG_ERR_UNSUPPORTED, "index_dtype must be F16, BF16 or F32");
+    if (M < 0) return fail(PRECOG_ERR_INVALID_ARG, "M must be >= 0");
+    if (M >= 0x7fffffffLL) return fail(PRECOG_ERR_UNSUPPORTED, "M must be below 2^31-1");
+    if (dim < 1) return fail(PRECOG_ERR_INVALID_ARG, "dim must be >= 1");
+    if ((static_cast<int64_t>(dim) * sz) % 16 != 0)
+        return fail(PRECOG_ERR_UNSUPPORTED, "dim*sizeof(dtype) must be a multiple of 16");
+    if (dim > 4096) return fail(PRECOG_ERR_UNSUPPORTED, "dim > 4096 is not implemented");
+    if (n_queries < 0) return fail(PRECOG_ERR_INVALID_ARG, "n_queries must be >= 0");
+    if (n_queries == 0) return ok();
+    if ((M > 0 && index == nullptr) || queries == nullptr || d_best_idx == nullptr)
+        return fail(PRECOG_ERR_INVALID_ARG, "index, queries and d_best_idx must be non-NULL");
+    if ((index && !aligned16(index)) || !aligned16(queries))
+        return fail(PRECOG_ERR_INVALID_ARG, "index and queries must be 16-byte aligned");
+    const size_t need = precog::retrieve_workspace_size(M, dim, n_queries);
+    if (workspace_bytes < need || (need > 0 && (workspace == nullptr || !aligned16(workspace))))
+        return fail(PRECOG_ERR_INVALID_ARG, "workspace too small or misaligned (%zu bytes needed)", need);
+    precog::RetrieveParams p;
+    p.index = index;
+    p.dtype = index_dtype;
+    p.M = M;
+    p.dim = dim;
+    p.queries = queries;
+    p.n_queries = n_queries;
+    p.best_idx = d_best_idx;
+    p.best_score = d_best_score;
+    p.workspace = workspace;
+    p.workspace_bytes = workspace_bytes;
+    cudaError_t e = precog::launch_retrieve(p, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "retrieve launch");
+    return ok();
+}
+
+precog_status precog_device_status(void *stream, uint32_t *bits_out) {
+    if (bits_out == nullptr) return fail(PRECOG_ERR_INVALID_ARG, "bits_out is NULL");
+    *bits_out = 0;
+    cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+    uint32_t a = 0, b = 0;
+    e = precog::scan_status_word_read_clear(&a);
+    if (e != cudaSuccess) return cuda_fail(e, "read scan status");
+    e = precog::retrieve_status_word_read_clear(&b);
+    if (e != cudaSuccess) return cuda_fail(e, "read retrieve status");
+    *bits_out = a | b;
+    if (*bits_out == 0) return ok();
+    if (*bits_out & PRECOG_DEV_TIMEOUT)
+        return fail(PRECOG_ERR_TIMEOUT, "a device-side wait gave up (bits 0x%x)", *bits_out);
+    return fail(PRECOG_ERR_DEVICE, "device flagged invalid offsets or bank rows (bits 0x%x)", *bits_out);
+}
+
+const char *precog_status_string(int32_t status) {
+    switch (status) {
+        case PRECOG_OK: return "PRECOG_OK";
+        case PRECOG_ERR_INVALID_ARG: return "PRECOG_ERR_INVALID_ARG";
+        case PRECOG_ERR_UNSUPPORTED: return "PRECOG_ERR_UNSUPPORTED";
+        case PRECOG_ERR_CUDA: return "PRECOG_ERR_CUDA";
+        case PRECOG_ERR_TIMEOUT: return "PRECOG_ERR_TIMEOUT";
+        case PRECOG_ERR_DEVICE: return "PRECOG_ERR_DEVICE";
+        default: return "PRECOG_UNKNOWN_STATUS";
+    }
+}
+
+const char *precog_last_error(void) { return g_last_error; }
+
+int32_t precog_abi_version(void) { return PRECOG_ABI_VERSION; }
+
+}  // extern "C"

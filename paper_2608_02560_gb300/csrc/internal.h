@@ -1,0 +1,61 @@
+// Host-side interfaces between the C ABI (api.cu) and the kernel files.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace precog {
+
+// One scan launch: L layers x n_chunks chunks x channel slices, each work item
+// a CTA that rolls the recurrence over one chunk for one slice of channels.
+struct ScanParams {
+    // inputs
+    const void *x, *dt, *B, *C;
+    const float *A;
+    int64_t ls_xd, ls_bc;     // layer strides in elements
+    int32_t n_layers, D, N;
+    int32_t in_dtype;         // precog_dtype
+    int64_t T_tot;            // rows per layer
+    // chunking: use_fixed -> chunk c is rows [c*fixed_len, (c+1)*fixed_len),
+    // else rows [offsets[c], offsets[c+1])
+    const int64_t *offsets;
+    int64_t n_chunks;
+    int32_t use_fixed;
+    int32_t fixed_len;
+    // initial state (prefill); bank == nullptr -> zero state
+    const void *bank;
+    int32_t bank_dtype;
+    int64_t bank_entries;
+    const int64_t *idx;       // nullptr -> row = chunk
+    int32_t L_bank;           // layers per bank entry
+    // outputs
+    void *states;             // [n_chunks][L_out][D][N] or nullptr
+    int32_t state_dtype;
+    int32_t L_out;            // layers per output entry
+    int32_t layer0;           // first layer of the bank / output entries
+    void *y;                  // [L][T_tot][D] or nullptr
+    int32_t y_dtype;
+};
+
+cudaError_t launch_scan(const ScanParams &p, cudaStream_t stream);
+cudaError_t scan_status_word_read_clear(uint32_t *bits);
+
+struct RetrieveParams {
+    const void *index;
+    int32_t dtype;
+    int64_t M;
+    int32_t dim;
+    const void *queries;
+    int32_t n_queries;
+    int64_t *best_idx;
+    float *best_score;
+    void *workspace;
+    size_t workspace_bytes;
+};
+
+size_t retrieve_workspace_size(int64_t M, int32_t dim, int32_t n_queries);
+cudaError_t launch_retrieve(const RetrieveParams &p, cudaStream_t stream);
+cudaError_t retrieve_status_word_read_clear(uint32_t *bits);
+
+}  // namespace precog

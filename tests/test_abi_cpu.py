@@ -1,0 +1,114 @@
+"""The C-ABI library loads and exports every symbol include/precog.h declares, and its
+host-side argument checks return the documented status codes without touching a GPU
+(no pointer passed here is ever dereferenced on the host)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "precog.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_02560_gb300 import build
+    build.build()
+    import paper_2608_02560_gb300 as pg
+    return pg.load_library()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(precog_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_header_declares_the_three_calls():
+    names = declared_functions()
+    for n in ("precog_encode_chunks", "precog_retrieve", "precog_prefill_from_state"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert len(names) >= 8
+    for n in names:
+        assert hasattr(lib, n), f"{n} declared in include/precog.h but not exported"
+
+
+def test_abi_version_and_status_strings(lib):
+    assert lib.precog_abi_version() == 1
+    for code, name in [(0, b"PRECOG_OK"), (1, b"PRECOG_ERR_INVALID_ARG"),
+                       (2, b"PRECOG_ERR_UNSUPPORTED"), (3, b"PRECOG_ERR_CUDA"),
+                       (4, b"PRECOG_ERR_TIMEOUT"), (5, b"PRECOG_ERR_DEVICE")]:
+        assert lib.precog_status_string(code) == name
+
+
+FAKE = 0x10000  # a 16-byte aligned address that the host never dereferences
+
+
+def _inputs(pg, **kw):
+    s = pg.ScanInputs()
+    s.n_layers, s.D, s.N, s.in_dtype = 1, 64, 16, pg.PRECOG_BF16
+    s.x = s.dt = s.B = s.C = s.A = FAKE
+    s.layer_stride_xd = s.layer_stride_bc = 0
+    for k, v in kw.items():
+        setattr(s, k, v)
+    return s
+
+
+def _encode(lib, s, offsets=FAKE, n_chunks=4, T_tot=64, states=FAKE, sdt=0, layer0=0, L=1,
+            y=None, ydt=0):
+    return lib.precog_encode_chunks(ctypes.byref(s) if s is not None else None, offsets, n_chunks,
+                                    T_tot, states, sdt, layer0, L, y, ydt, None)
+
+
+@pytest.mark.parametrize("change,expect", [
+    ({"N": 8}, 2), ({"D": 0}, 1), ({"D": 12}, 2), ({"in_dtype": 2}, 2), ({"x": 0}, 1),
+    ({"A": FAKE + 4}, 1), ({"n_layers": 0}, 1), ({"n_layers": 2, "layer_stride_xd": 10}, 1),
+])
+def test_encode_rejects_bad_inputs(lib, change, expect):
+    import paper_2608_02560_gb300 as pg
+    assert _encode(lib, _inputs(pg, **change)) == expect
+    assert lib.precog_last_error() != b""
+
+
+def test_encode_rejects_bad_call_arguments(lib):
+    import paper_2608_02560_gb300 as pg
+    s = _inputs(pg)
+    assert _encode(lib, None) == 1
+    assert _encode(lib, s, offsets=None) == 1
+    assert _encode(lib, s, n_chunks=-1) == 1
+    assert _encode(lib, s, T_tot=-5) == 1
+    assert _encode(lib, s, states=None, y=None) == 1
+    assert _encode(lib, s, sdt=2) == 2                      # fp16 states unsupported
+    assert _encode(lib, s, layer0=1, L=1) == 1              # layer outside the bank entry
+    assert _encode(lib, s, states=FAKE + 8) == 1            # misaligned output
+    assert _encode(lib, _inputs(pg, C=None), y=FAKE) == 1   # readout needs C
+    assert _encode(lib, s, n_chunks=0) == 0                 # nothing to do: OK, no launch
+
+
+def test_prefill_rejects_bad_arguments(lib):
+    import paper_2608_02560_gb300 as pg
+    s = _inputs(pg)
+    f = lib.precog_prefill_from_state
+    assert f(ctypes.byref(s), 1, 4, None, 1, 10, 24, 0, FAKE, FAKE, 0, FAKE, 0, None) == 1
+    assert f(ctypes.byref(s), 1, 4, FAKE, 1, 10, 24, 24, FAKE, FAKE, 0, FAKE, 0, None) == 1
+    assert f(ctypes.byref(s), 3, 4, FAKE, 1, 2, 24, 0, None, FAKE, 0, FAKE, 0, None) == 1
+    assert f(ctypes.byref(s), 1, 4, FAKE, 1, 10, 24, 0, FAKE, None, 0, None, 0, None) == 1
+    assert f(ctypes.byref(s), -1, 4, FAKE, 1, 10, 24, 0, FAKE, FAKE, 0, FAKE, 0, None) == 1
+    assert f(ctypes.byref(s), 0, 4, FAKE, 1, 10, 24, 0, FAKE, FAKE, 0, FAKE, 0, None) == 0
+
+
+def test_retrieve_rejects_bad_arguments(lib):
+    f = lib.precog_retrieve
+    assert f(FAKE, 2, 100, 768, FAKE, 1, FAKE, FAKE, FAKE, 0, None) == 1       # no workspace
+    assert f(FAKE, 2, 100, 12, FAKE, 1, FAKE, FAKE, FAKE, 1 << 20, None) == 2   # 24 B rows
+    assert f(FAKE, 7, 100, 768, FAKE, 1, FAKE, FAKE, FAKE, 1 << 20, None) == 2  # dtype
+    assert f(FAKE, 2, -1, 768, FAKE, 1, FAKE, FAKE, FAKE, 1 << 20, None) == 1
+    assert f(FAKE, 2, 1 << 31, 768, FAKE, 1, FAKE, FAKE, FAKE, 1 << 40, None) == 2
+    assert f(FAKE, 2, 100, 768, None, 1, FAKE, FAKE, FAKE, 1 << 20, None) == 1
+    assert f(FAKE, 2, 100, 768, FAKE, 0, FAKE, FAKE, FAKE, 0, None) == 0       # no queries
+    assert lib.precog_retrieve_workspace_size(100, 768, 4) >= 4 * 8

@@ -1,0 +1,140 @@
+"""GPU parity of state injection + query prefill (Eq. 2) and Theorem 1 through the C ABI."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from tests._util import TOL_BF16, TOL_F32, rel_err, rel_err_stored, to_np
+
+pytestmark = pytest.mark.gpu
+
+
+def _pg():
+    import paper_2608_02560_gb300 as pg
+    return pg
+
+
+def _t(a, dev, dtype=None):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(a)).to(dev, dtype or torch.float32)
+
+
+def test_theorem1_via_abi_bit_identical(cuda_device):
+    """Encode [chunk; query] from the zero state with readout, versus encode(chunk) then
+    prefill(query) from the captured fp32 state: identical operation sequence on the GPU,
+    so states and every query y_t agree bit for bit (Theorem 1, Proposition)."""
+    import torch
+    pg = _pg()
+    d = cuda_device
+    D, N = 256, 16
+    Lc, Tq = 413, 64
+    x, dt, A, B, C = synth.host_scan_inputs(Lc + Tq, D, N, seed=123)
+    tb = lambda a: _t(a, d, torch.bfloat16)
+    xb, dtb, Bb, Cb, Ad = tb(x), tb(dt), tb(B), tb(C), _t(A, d)
+    full_state = torch.empty((1, 1, D, N), dtype=torch.float32, device=d)
+    full_y = torch.empty((1, Lc + Tq, D), dtype=torch.float32, device=d)
+    pg.precog_encode_chunks(pg.scan_inputs(xb, dtb, Bb, Ad, Cb),
+                            _t(np.array([0, Lc + Tq]), d, torch.int64), Lc + Tq,
+                            states_out=full_state, y_out=full_y)
+    ctx_state = torch.empty((1, 1, D, N), dtype=torch.float32, device=d)
+    pg.precog_encode_chunks(pg.scan_inputs(xb[:Lc], dtb[:Lc], Bb[:Lc], Ad),
+                            _t(np.array([0, Lc]), d, torch.int64), Lc, states_out=ctx_state)
+    q_y = torch.empty((1, Tq, D), dtype=torch.float32, device=d)
+    q_state = torch.empty((1, 1, D, N), dtype=torch.float32, device=d)
+    pg.precog_prefill_from_state(pg.scan_inputs(xb[Lc:].contiguous(), dtb[Lc:].contiguous(),
+                                                Bb[Lc:].contiguous(), Ad, Cb[Lc:].contiguous()),
+                                 1, Tq, ctx_state, idx=None, y_out=q_y, state_out=q_state)
+    assert pg.precog_device_status()[0] == 0
+    assert torch.equal(full_state, q_state)
+    assert torch.equal(full_y[:, Lc:], q_y)
+    # and both agree with the oracle's in-context scan
+    ref_h, ref_y = oracle.rollout(to_np(xb), to_np(dtb), A, to_np(Bb), to_np(Cb), want_y=True)
+    assert rel_err(to_np(q_state[0, 0]), ref_h) < 1e-5
+    assert rel_err(to_np(q_y[0]), ref_y[Lc:]) < 1e-5
+
+
+def test_tiny_end_to_end(cuda_device):
+    """Encode 8 chunks, retrieve for the planted query, inject, prefill 32 tokens; compare
+    with the oracle scanning [chunk 3; query] from the zero state."""
+    import torch
+    pg = _pg()
+    d = cuda_device
+    w = synth.tiny_workload(0)
+    D, N = w.A.shape
+    bank = torch.empty((8, 1, D, N), dtype=torch.float32, device=d)
+    pg.precog_encode_chunks(pg.scan_inputs(_t(w.x, d), _t(w.dt, d), _t(w.B, d), _t(w.A, d)),
+                            _t(w.offsets, d, torch.int64), w.x.shape[0], states_out=bank)
+    idx = torch.empty(1, dtype=torch.int64, device=d)
+    pg.precog_retrieve(_t(w.index, d), _t(w.query, d), idx)
+    y = torch.empty((1, 32, D), dtype=torch.float32, device=d)
+    h = torch.empty((1, 1, D, N), dtype=torch.float32, device=d)
+    pg.precog_prefill_from_state(pg.scan_inputs(_t(w.qx, d), _t(w.qdt, d), _t(w.qB, d),
+                                                _t(w.A, d), _t(w.qC, d)),
+                                 1, 32, bank, idx=idx, y_out=y, state_out=h)
+    assert pg.precog_device_status()[0] == 0
+    assert int(idx.item()) == w.planted
+    s, e = w.offsets[w.planted], w.offsets[w.planted + 1]
+    cat = lambda a, b: np.vstack([a[s:e], b])
+    ref_h, ref_y = oracle.rollout(cat(w.x, w.qx), cat(w.dt, w.qdt), w.A, cat(w.B, w.qB),
+                                  cat(w.C, w.qC), want_y=True)
+    assert rel_err(to_np(h[0, 0]), ref_h) < TOL_F32
+    assert rel_err(to_np(y[0]), ref_y[e - s:]) < TOL_F32
+
+
+def test_bad_and_missing_rows(cuda_device):
+    """idx = -1 injects the zero state (no retrieved context, no flag); a row beyond the
+    bank injects zeros and flags PRECOG_DEV_BAD_INDEX; T_q = 0 returns the injected state."""
+    import torch
+    pg = _pg()
+    d = cuda_device
+    D, N, T = 64, 16, 20
+    x, dt, A, B, C = synth.host_scan_inputs(3 * T, D, N, seed=5)
+    bank = torch.randn((4, 2, D, N), device=d)
+    idx = torch.tensor([-1, 2, 99], dtype=torch.int64, device=d)
+    h = torch.empty((3, 2, D, N), dtype=torch.float32, device=d)
+    inputs = pg.scan_inputs(_t(x, d), _t(dt, d), _t(B, d), _t(A, d))
+    pg.precog_prefill_from_state(inputs, 3, T, bank, idx=idx, layer0=1, state_out=h)
+    st, bits = pg.precog_device_status()
+    assert st == 5 and bits == pg.PRECOG_DEV_BAD_INDEX
+    for q, h0 in ((0, None), (1, to_np(bank[2, 1])), (2, None)):
+        sl = slice(q * T, (q + 1) * T)
+        ref, _ = oracle.rollout(x[sl], dt[sl], A, B[sl], h0=h0)
+        assert rel_err(to_np(h[q, 1]), ref) < TOL_F32
+    h2 = torch.empty((3, 2, D, N), dtype=torch.float32, device=d)
+    empty = pg.scan_inputs(_t(x[:0], d), _t(dt[:0], d), _t(B[:0], d), _t(A, d))
+    pg.precog_prefill_from_state(empty, 3, 0, bank, idx=idx[1:2].repeat(3), layer0=1, state_out=h2)
+    assert pg.precog_device_status()[0] == 0
+    assert torch.equal(h2[:, 1], bank[2, 1].expand(3, D, N))
+
+
+@pytest.mark.parametrize("Q", [1, 256])
+def test_query_workload_prefill(cuda_device, Q):
+    """Query-time path at full per-query size: inject a 24-layer (D=256, N=16) bf16 state
+    gathered through device-resident indices and prefill 64 bf16 tokens per query, in the
+    launch configuration the benchmark times. Sampled (query, layer) pairs vs the oracle."""
+    import torch
+    pg = _pg()
+    d = cuda_device
+    L, D, N, Tq = 24, 256, 16, synth.QUERY_TOKENS
+    entries = 4096
+    bank = synth.device_normal_bank(entries, L * D * N, 1, d).view(entries, L, D, N)
+    g = torch.Generator(device=d)
+    g.manual_seed(Q)
+    idx = torch.randint(0, entries, (Q,), generator=g, device=d)
+    ins = [synth.device_scan_inputs(Q * Tq, D, N, 2, l, d) for l in range(L)]
+    stack = lambda k: torch.stack([i[k] for i in ins]).contiguous()
+    x, dt, B, C, A = stack("x"), stack("dt"), stack("B"), stack("C"), stack("A")
+    y = torch.empty((L, Q * Tq, D), dtype=torch.bfloat16, device=d)
+    h = torch.empty((Q, L, D, N), dtype=torch.bfloat16, device=d)
+    pg.precog_prefill_from_state(pg.scan_inputs(x, dt, B, A, C), Q, Tq, bank, idx=idx,
+                                 y_out=y, state_out=h)
+    assert pg.precog_device_status()[0] == 0
+    An = A[0].cpu().numpy()
+    for q in sorted({0, Q - 1, Q // 3}):
+        for l in (0, 13, 23):
+            sl = slice(q * Tq, (q + 1) * Tq)
+            h0 = to_np(bank[idx[q].item(), l])
+            ref_h, ref_y = oracle.rollout(to_np(x[l, sl]), to_np(dt[l, sl]), An, to_np(B[l, sl]),
+                                          to_np(C[l, sl]), h0=h0, want_y=True)
+            assert rel_err_stored(to_np(h[q, l]), ref_h) < TOL_BF16
+            assert rel_err_stored(to_np(y[l, sl]), ref_y) < TOL_BF16

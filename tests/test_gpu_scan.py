@@ -1,0 +1,240 @@
+"""GPU parity of the scan kernel (encode with state capture, readout y) against the oracle.
+
+Called through the C ABI. Small cases are compared element by element; the full-size
+workloads (single-layer wide encode, paper-shaped encode, ragged large-scale encode) run
+in the launch configuration the benchmark times, and sampled chunks are compared with
+the oracle one by one on inputs copied back from the device generator.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from tests._util import TOL_BF16, TOL_F32, rel_err, rel_err_stored, to_np
+
+pytestmark = pytest.mark.gpu
+
+
+def _pg():
+    import paper_2608_02560_gb300 as pg
+    return pg
+
+
+def _t(a, dev, dtype=None):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(a)).to(dev, dtype or torch.float32)
+
+
+def _encode(dev, x, dt, B, A, offsets, C=None, state_dtype=None, y_dtype=None):
+    import torch
+    pg = _pg()
+    n_chunks = offsets.numel() - 1
+    L = 1 if x.dim() == 2 else x.shape[0]
+    D, N = A.shape[-2], A.shape[-1]
+    states = torch.full((n_chunks, L, D, N), float("nan"), dtype=state_dtype or torch.float32,
+                        device=dev)
+    y = None
+    if y_dtype is not None:
+        T = x.shape[-2]
+        y = torch.zeros((L, T, D), dtype=y_dtype, device=dev)
+    pg.precog_encode_chunks(pg.scan_inputs(x, dt, B, A, C), offsets, x.shape[-2], states_out=states,
+                            y_out=y)
+    st, bits = pg.precog_device_status()
+    assert st == 0, f"device status {st} bits {bits:#x}"
+    return states, y
+
+
+def test_tiny_workload_fp32(cuda_device):
+    """1 layer, D=64, N=16, fp32, 8 chunks x 256 tokens: states and every y_t."""
+    import torch
+    w = synth.tiny_workload(0)
+    d = cuda_device
+    states, y = _encode(d, _t(w.x, d), _t(w.dt, d), _t(w.B, d), _t(w.A, d),
+                        _t(w.offsets, d, torch.int64), C=_t(w.C, d), y_dtype=torch.float32)
+    ref_s, ref_y = oracle.scan(w.x, w.dt, w.A, w.B, w.offsets, C=w.C, want_y=True)
+    for c in range(ref_s.shape[0]):
+        assert rel_err(to_np(states[c, 0]), ref_s[c]) < TOL_F32
+        s, e = w.offsets[c], w.offsets[c + 1]
+        assert rel_err(to_np(y[0, s:e]), ref_y[s:e]) < TOL_F32
+
+
+@pytest.mark.parametrize("D,lens", [(64, [1, 15, 16, 17, 0, 300]), (96, [40, 33]),
+                                    (8, [5, 100]), (512, [70, 0, 2])])
+def test_ragged_lengths_and_widths_generic_A(cuda_device, D, lens):
+    """Unstructured A (one exponential per (d, n)), ragged tails, empty chunks, widths
+    that need several channel slices or fewer than a warp of threads."""
+    import torch
+    d = cuda_device
+    N = 16
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    T = int(off[-1])
+    x, dt, _, B, C = synth.host_scan_inputs(T, D, N, seed=D + len(lens))
+    A = -np.random.default_rng(D).uniform(0.05, 3.0, size=(D, N)).astype(np.float32)
+    states, y = _encode(d, _t(x, d), _t(dt, d), _t(B, d), _t(A, d), _t(off, d, torch.int64),
+                        C=_t(C, d), y_dtype=torch.float32)
+    ref_s, ref_y = oracle.scan(x, dt, A, B, off, C=C, want_y=True)
+    for c in range(len(lens)):
+        if lens[c] == 0:
+            assert np.all(to_np(states[c, 0]) == 0)
+            continue
+        assert rel_err(to_np(states[c, 0]), ref_s[c]) < TOL_F32
+        assert rel_err(to_np(y[0, off[c]:off[c + 1]]), ref_y[off[c]:off[c + 1]]) < TOL_F32
+
+
+def test_A_zero_cumulative_sum_bit_exact(cuda_device):
+    """A = 0: alpha = 1 exactly and h is a running sum. Dyadic inputs keep every fp32
+    product and sum exact, so the GPU must match the exact cumulative sum bit for bit."""
+    import torch
+    d = cuda_device
+    rng = np.random.default_rng(3)
+    T, D, N = 200, 64, 16
+    x = (rng.integers(-8, 9, size=(T, D)) / 8.0).astype(np.float32)
+    dt = (rng.integers(1, 5, size=(T, D)) / 4.0).astype(np.float32)
+    B = (rng.integers(-4, 5, size=(T, N)) / 4.0).astype(np.float32)
+    C = (rng.integers(-4, 5, size=(T, N)) / 4.0).astype(np.float32)
+    A = np.zeros((D, N), dtype=np.float32)
+    off = np.array([0, 77, T], dtype=np.int64)
+    states, y = _encode(d, _t(x, d), _t(dt, d), _t(B, d), _t(A, d), _t(off, d, torch.int64),
+                        C=_t(C, d), y_dtype=torch.float32)
+    for c in range(2):
+        s, e = off[c], off[c + 1]
+        traj = np.cumsum((dt[s:e] * x[s:e]).astype(np.float64)[:, :, None] * B[s:e, None, :], axis=0)
+        np.testing.assert_array_equal(to_np(states[c, 0]), traj[-1])
+        np.testing.assert_array_equal(to_np(y[0, s:e]), np.einsum("tn,tdn->td", C[s:e], traj))
+
+
+def test_multi_layer_call_and_layer_offset(cuda_device):
+    """Three layers in one call with independent inputs, written at layer0=2 of a
+    5-layer bank entry; the other layers stay untouched."""
+    import torch
+    pg = _pg()
+    d = cuda_device
+    L, T, D, N = 3, 96, 64, 16
+    lens = [30, 66]
+    off = np.array([0, 30, 96], dtype=np.int64)
+    ins = [synth.host_scan_inputs(T, D, N, seed=50 + l) for l in range(L)]
+    x = _t(np.stack([i[0] for i in ins]), d)
+    dt = _t(np.stack([i[1] for i in ins]), d)
+    B = _t(np.stack([i[3] for i in ins]), d)
+    A = _t(np.stack([synth.structured_A(D, N) * (1 + 0.5 * l) for l in range(L)]), d)
+    bank = torch.full((2, 5, D, N), 7.0, dtype=torch.float32, device=d)
+    pg.precog_encode_chunks(pg.scan_inputs(x, dt, B, A), _t(off, d, torch.int64), T,
+                            states_out=bank, layer0=2, L_total=5)
+    assert pg.precog_device_status()[0] == 0
+    got = to_np(bank)
+    assert np.all(got[:, :2] == 7.0)
+    for l in range(L):
+        ref, _ = oracle.scan(ins[l][0], ins[l][1], synth.structured_A(D, N) * (1 + 0.5 * l),
+                             ins[l][3], off)
+        for c in range(2):
+            assert rel_err(got[c, 2 + l], ref[c]) < TOL_F32
+
+
+def test_bf16_capture_and_readout(cuda_device):
+    """bf16 inputs, fp32 accumulation: bf16 and fp32 state capture, bf16 readout."""
+    import torch
+    d = cuda_device
+    T, D, N = 700, 256, 16
+    off = np.array([0, 300, 301, 700], dtype=np.int64)
+    x, dt, A, B, C = synth.host_scan_inputs(T, D, N, seed=77)
+    tb = lambda a: _t(a, d, torch.bfloat16)
+    xb, dtb, Bb, Cb = tb(x), tb(dt), tb(B), tb(C)
+    s16, y16 = _encode(d, xb, dtb, Bb, _t(A, d), _t(off, d, torch.int64), C=Cb,
+                       state_dtype=torch.bfloat16, y_dtype=torch.bfloat16)
+    s32, _ = _encode(d, xb, dtb, Bb, _t(A, d), _t(off, d, torch.int64))
+    ref_s, ref_y = oracle.scan(to_np(xb), to_np(dtb), A, to_np(Bb), off, C=to_np(Cb), want_y=True)
+    for c in range(3):
+        assert rel_err(to_np(s32[c, 0]), ref_s[c]) < 1e-5
+        assert rel_err_stored(to_np(s16[c, 0]), ref_s[c]) < TOL_BF16
+        sl = slice(off[c], off[c + 1])
+        assert rel_err_stored(to_np(y16[0, sl]), ref_y[sl]) < TOL_BF16
+
+
+def test_bad_offsets_flag_device_status(cuda_device):
+    """Non-monotone or out-of-range offsets are skipped and reported, never faulted."""
+    import torch
+    pg = _pg()
+    d = cuda_device
+    T, D, N = 64, 64, 16
+    x, dt, A, B, _ = synth.host_scan_inputs(T, D, N, seed=1)
+    off = _t(np.array([0, 40, 20, 64, 1000], dtype=np.int64), d, torch.int64)
+    states = torch.zeros((4, 1, D, N), dtype=torch.float32, device=d)
+    pg.precog_encode_chunks(pg.scan_inputs(_t(x, d), _t(dt, d), _t(B, d), _t(A, d)), off, T,
+                            states_out=states)
+    st, bits = pg.precog_device_status()
+    assert st == 5 and bits & pg.PRECOG_DEV_BAD_OFFSETS
+    assert pg.precog_device_status() == (0, 0)   # the word was cleared
+    ref, _ = oracle.scan(x, dt, A, B, np.array([0, 40], dtype=np.int64))
+    assert rel_err(to_np(states[0, 0]), ref[0]) < TOL_F32
+
+
+def test_deterministic(cuda_device):
+    import torch
+    d = cuda_device
+    x, dt, A, B, _ = synth.host_scan_inputs(512, 256, 16, seed=9)
+    off = _t(np.array([0, 256, 512], dtype=np.int64), d, torch.int64)
+    args = [_t(v, d, torch.bfloat16) for v in (x, dt, B)]
+    a, _ = _encode(d, args[0], args[1], args[2], _t(A, d), off)
+    b, _ = _encode(d, args[0], args[1], args[2], _t(A, d), off)
+    assert torch.equal(a, b)
+
+
+# ------------------------------------------------------------- full-size workloads, sampled
+
+
+def _sampled_check(dev, shape, layer, sample_chunks, y_mode=False, seed=0):
+    """Generate one layer of a workload on the device at full size, run the encode as the
+    benchmark does, copy back the sampled chunks' inputs and compare with the oracle."""
+    import torch
+    pg = _pg()
+    off_np = synth.shape_offsets(shape, seed)
+    T = int(off_np[-1])
+    inp = synth.device_scan_inputs(T, shape.D, shape.N, seed, layer, dev, with_C=y_mode)
+    off = torch.from_numpy(off_np).to(dev)
+    states = torch.empty((shape.n_chunks, shape.n_layers, shape.D, shape.N), dtype=torch.bfloat16,
+                         device=dev)
+    y = torch.empty((1, T, shape.D), dtype=torch.bfloat16, device=dev) if y_mode else None
+    pg.precog_encode_chunks(pg.scan_inputs(inp["x"], inp["dt"], inp["B"], inp["A"],
+                                           inp.get("C") if y_mode else None),
+                            off, T, states_out=states, layer0=layer, L_total=shape.n_layers,
+                            y_out=y)
+    assert pg.precog_device_status()[0] == 0
+    A = inp["A"].cpu().numpy()
+    worst = 0.0
+    for c in sample_chunks:
+        s, e = int(off_np[c]), int(off_np[c + 1])
+        xs = to_np(inp["x"][s:e])
+        dts = to_np(inp["dt"][s:e])
+        Bs = to_np(inp["B"][s:e])
+        Cs = to_np(inp["C"][s:e]) if y_mode else None
+        ref_h, ref_y = oracle.rollout(xs, dts, A, Bs, Cs, want_y=y_mode)
+        err = rel_err_stored(to_np(states[c, layer]), ref_h)
+        worst = max(worst, err)
+        assert err < TOL_BF16, (c, err)
+        if y_mode:
+            assert rel_err_stored(to_np(y[0, s:e]), ref_y) < TOL_BF16
+    del inp, states, y
+    torch.cuda.empty_cache()
+    return worst
+
+
+def test_wide_single_layer_full_size(cuda_device):
+    """1 layer, D=2048, N=16, 1024 chunks x 512 tokens, bf16 (capture and y modes)."""
+    _sampled_check(cuda_device, synth.WIDE, 0, [0, 511, 1023])
+    _sampled_check(cuda_device, synth.WIDE, 0, [3, 1000], y_mode=True)
+
+
+def test_paper_shaped_encode_full_size(cuda_device):
+    """24 x (D=256, N=16) layers, 4096 chunks x 3000 tokens, bf16: layers 0 and 23 at
+    full size into the 192 KB-per-chunk bf16 bank layout."""
+    _sampled_check(cuda_device, synth.PAPER, 0, [0, 2047, 4095])
+    _sampled_check(cuda_device, synth.PAPER, 23, [1, 4094])
+
+
+def test_ragged_large_scale_encode_full_size(cuda_device):
+    """8192 ragged chunks (lengths 256..4096), D=512, N=16, bf16: the longest, the
+    shortest and a few random chunks of one layer."""
+    off = synth.shape_offsets(synth.RAGGED, 0)
+    lens = np.diff(off)
+    pick = sorted({int(np.argmax(lens)), int(np.argmin(lens)), 0, 4097, 8191})
+    _sampled_check(cuda_device, synth.RAGGED, 5, pick)

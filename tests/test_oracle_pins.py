@@ -284,3 +284,16 @@ def test_paper_state_size():
     # the paper-shaped workload stores the same 192 KB: 24 layers x D=256 x N=16 x 2 B
     s = synth.PAPER
     assert s.n_layers * s.D * s.N * 2 == g["total_state_bytes"]
+
+
+def test_bf16_storage_tolerance_helper():
+    """The comparison used for bf16-stored outputs allows exactly the one rounding:
+    torch's round-to-nearest-even bf16 cast of the exact value scores 0."""
+    import torch
+    from tests._util import rel_err_stored
+    ref = np.random.default_rng(0).standard_normal(10000) * 3.0
+    stored = torch.from_numpy(ref).to(torch.bfloat16).double().numpy()
+    assert rel_err_stored(stored, ref) == 0.0
+    bumped = stored.copy()
+    bumped[np.argmax(np.abs(ref))] *= 1 + 2.0 ** -6         # two ulps off at the maximum
+    assert rel_err_stored(bumped, ref) > 2e-3
