@@ -1,0 +1,511 @@
+#!/usr/bin/env python
+"""PRECOG hot-path benchmark on GB300.
+
+One step = one pass of the whole hot path over one batch of synthetic input:
+  * corpus encode of the paper-shaped workload: 24 independent layers (D=256,
+    N=16), 4096 chunks x 3000 tokens, bf16 inputs, fp32 state, captured into a
+    bf16 bank of 192 KB per chunk (24 C-ABI encode calls, one per layer);
+  * the query-time path: top-1 retrieval of a query batch over 1,000,000
+    unit-norm fp16 keys of dim 768, injection of the retrieved 192 KB state from
+    a 1,000,000-entry bank and scan prefill of 64 query tokens per query.
+
+value = corpus tokens encoded per second (through all 24 layers) by all ranks.
+The 24 layers' inputs (12.98 GB each, 311 GB in all) exceed HBM: `--input-sets`
+independently generated layer inputs stay resident and layer l reads set
+l mod S. Every encode call still streams its full 12.98 GB from HBM (far above
+the 129 MB L2), so the timed traffic and work equal those of 24 independent
+layers; generating the synthetic inputs is not part of the method and is
+timed separately. The retrieve+inject+prefill p50 latency is measured after the
+timed steps, per query batch, with an L2 flush before every iteration.
+
+`--impl reference` times the CPU oracle (fp64, sequential) on a bounded sample
+of the same workload on the host cores and prints the same JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "corpus-encode tokens/s & % HBM roofline; retrieve+inject+prefill p50 latency"
+UNIT = "tokens/s"
+FALLBACK_HBM_GBS = 6800.0
+PROFILE = os.path.join(ROOT, "profiles", "scan_encode_paper_shaped.md")
+SCAN_SRC = os.path.join(ROOT, "paper_2608_02560_gb300", "csrc", "scan.cu")
+
+
+def parse_args():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--input-sets", type=int, default=2)
+    ap.add_argument("--query-batch", type=int, default=1)
+    ap.add_argument("--latency-iters", type=int, default=200)
+    ap.add_argument("--e2e-steps", type=int, default=2)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-latency", action="store_true")
+    ap.add_argument("--case", choices=["full", "scan-small", "retrieve-small", "prefill-small"],
+                    default="full",
+                    help="small single-kernel cases (a few GB) used for profiler captures")
+    return ap.parse_args()
+
+
+def scan_bytes_per_launch(T, n_chunks, D, N, in_bytes=2, state_bytes=2):
+    """Algorithmic HBM bytes of one encode launch: every input element read once
+    (x, dt: T*D each; B: T*N), the captured state written once, the offsets and A read."""
+    return T * (2 * D + N) * in_bytes + n_chunks * D * N * state_bytes + 8 * (n_chunks + 1) + 4 * D * N
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        try:
+            p = json.load(open(path))
+            return float(p["hbm_gbs"]), "measured"
+        except Exception:
+            pass
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+def profiled_traffic():
+    """Per-launch DRAM traffic from the committed ncu summary, if it was taken on the
+    current scan kernel source (else None)."""
+    if not os.path.exists(PROFILE):
+        return None
+    text = open(PROFILE).read()
+    m_sha = re.search(r"scan\.cu sha256:\s*([0-9a-f]{64})", text)
+    m_tr = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    if not m_sha or not m_tr:
+        return None
+    sha = hashlib.sha256(open(SCAN_SRC, "rb").read()).hexdigest()
+    return float(m_tr.group(1)) if sha == m_sha.group(1) else None
+
+
+class Clocks:
+    """Samples nvidia-smi clocks and throttle reasons while a region runs."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        if self.path and os.path.exists(self.path):
+            for line in open(self.path):
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+            os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        power = [float(r[3]) for r in rows if re.match(r"^[0-9.]+$", r[3])]
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "power_w_max": max(power) if power else None, "samples": len(rows)}
+
+
+# ------------------------------------------------------------------------------ reference arm
+
+
+def run_reference(args):
+    """The oracle (fp64, sequential, one host core) on a bounded sample of the encode."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import numpy as np
+    import torch
+
+    import oracle
+    import synth
+    shape = synth.PAPER
+    chunks, T = 1, shape.chunk_len
+    x, dt, A, B, _ = synth.host_scan_inputs(chunks * T, shape.D, shape.N, seed=0)
+    # bf16 inputs, widened exactly, as the GPU path sees them
+    bf = lambda a: torch.from_numpy(a).to(torch.bfloat16).double().numpy()
+    x, dt, B = bf(x), bf(dt), bf(B)
+    off = synth.fixed_offsets(chunks, T)
+    oracle.build()
+    for _ in range(args.warmup):
+        oracle.scan(x, dt, A, B, off)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oracle.scan(x, dt, A, B, off)
+        times.append(time.perf_counter() - t0)
+    per_layer = chunks * T / statistics.mean(times)
+    value = per_layer / shape.n_layers          # tokens through all 24 layers per second
+    sample = (f"{chunks} chunk x {T} tokens x 1 layer of the paper-shaped encode (D=256, N=16), "
+              f"bf16-valued inputs in fp64; rate divided by 24 layers")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * statistics.mean(times), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": "paper-shaped corpus encode (sampled for the CPU oracle)",
+                       "chunk_tokens": T, "layers": shape.n_layers, "D": shape.D, "N": shape.N},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------------------ profiler cases
+
+
+def run_case(args):
+    """Small cases of one kernel each, sized above L2 but a few GB on the device, for
+    profiler captures: 3 launches of the kernel (the first is a warm-up)."""
+    import torch
+
+    import paper_2608_02560_gb300 as pg
+    import synth
+    dev = torch.device("cuda:0")
+    res = {"case": args.case}
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
+    if args.case == "scan-small":
+        shape, chunks = synth.PAPER, 512
+        off_np = synth.fixed_offsets(chunks, shape.chunk_len)
+        T = int(off_np[-1])
+        inp = synth.device_scan_inputs(T, shape.D, shape.N, 0, 0, dev, with_C=False)
+        bank = torch.empty((chunks, shape.n_layers, shape.D, shape.N), dtype=torch.bfloat16, device=dev)
+        off = torch.from_numpy(off_np).to(dev)
+        si = pg.scan_inputs(inp["x"], inp["dt"], inp["B"], inp["A"], a_kind=pg.PRECOG_A_POWER)
+        fn = lambda: pg.precog_encode_chunks(si, off, T, states_out=bank, layer0=0, L_total=shape.n_layers)
+        res["algorithmic_bytes_per_launch"] = scan_bytes_per_launch(T, chunks, shape.D, shape.N)
+        res["scale_to_full_launch"] = shape.n_chunks / chunks
+    elif args.case == "retrieve-small":
+        M = 1 << 18
+        index = synth.device_unit_index(M, synth.QUERY_DIM, 0, dev)
+        q, _ = synth.device_planted_queries(index, args.query_batch, synth.QUERY_NOISE, 1)
+        idx = torch.empty(args.query_batch, dtype=torch.int64, device=dev)
+        fn = lambda: pg.precog_retrieve(index, q, idx)
+        res["algorithmic_bytes_per_launch"] = M * synth.QUERY_DIM * 2
+    else:
+        L, D, N, Tq, Q, entries = 24, 256, 16, synth.QUERY_TOKENS, args.query_batch, 4096
+        bank = synth.device_normal_bank(entries, L * D * N, 1, dev).view(entries, L, D, N)
+        ins = [synth.device_scan_inputs(Q * Tq, D, N, 2, l, dev) for l in range(L)]
+        st = lambda k: torch.stack([i[k] for i in ins]).contiguous()
+        x, dt, B, C, A = st("x"), st("dt"), st("B"), st("C"), st("A")
+        si = pg.scan_inputs(x, dt, B, A, C, a_kind=pg.PRECOG_A_POWER)
+        idx = torch.arange(Q, dtype=torch.int64, device=dev) * 7 % entries
+        y = torch.empty((L, Q * Tq, D), dtype=torch.bfloat16, device=dev)
+        h = torch.empty((Q, L, D, N), dtype=torch.bfloat16, device=dev)
+        fn = lambda: pg.precog_prefill_from_state(si, Q, Tq, bank, idx=idx, y_out=y, state_out=h)
+    times = []
+    for i in range(3):
+        ev[2 * i].record()
+        fn()
+        ev[2 * i + 1].record()
+    torch.cuda.synchronize()
+    res["ms"] = [ev[2 * i].elapsed_time(ev[2 * i + 1]) for i in range(3)]
+    st, bits = pg.precog_device_status()
+    res["device_status"] = [st, bits]
+    print(json.dumps(res), flush=True)
+    if st != 0:
+        sys.exit(1)
+
+
+# ------------------------------------------------------------------------------ our arm
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+        return
+    if args.case != "full":
+        run_case(args)
+        return
+    import torch
+
+    import paper_2608_02560_gb300 as pg
+    import synth
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    pg.load_library()
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+
+    def max_over_ranks(v):
+        if world == 1:
+            return v
+        t = torch.tensor([v], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        return float(t.item())
+
+    shape = synth.PAPER
+    L, D, N = shape.n_layers, shape.D, shape.N
+    seed = 1000 * rank
+    off_np = synth.shape_offsets(shape, seed)
+    T = int(off_np[-1])
+    off = torch.from_numpy(off_np).to(dev)
+
+    t_gen = time.perf_counter()
+    sets = [synth.device_scan_inputs(T, D, N, seed, s, dev, with_C=False)
+            for s in range(args.input_sets)]
+    torch.cuda.synchronize()
+    gen_s_per_layer = (time.perf_counter() - t_gen) / args.input_sets
+    bank = torch.empty((shape.n_chunks, L, D, N), dtype=torch.bfloat16, device=dev)
+    scan_in = [pg.scan_inputs(s["x"], s["dt"], s["B"], s["A"], a_kind=pg.PRECOG_A_POWER) for s in sets]
+
+    # query-time workload
+    M, dim, Tq, Q = synth.QUERY_INDEX_M, synth.QUERY_DIM, synth.QUERY_TOKENS, args.query_batch
+    index = synth.device_unit_index(M, dim, seed + 1, dev)
+    qbank = synth.device_normal_bank(M, L * D * N, seed + 2, dev).view(M, L, D, N)
+
+    def query_batch(nq, qseed):
+        q, rows = synth.device_planted_queries(index, nq, synth.QUERY_NOISE, qseed)
+        ins = [synth.device_scan_inputs(nq * Tq, D, N, qseed, l, dev) for l in range(L)]
+        st = lambda k: torch.stack([i[k] for i in ins]).contiguous()
+        qx, qdt, qB, qC, qA = st("x"), st("dt"), st("B"), st("C"), st("A")
+        out = {"q": q, "rows": rows, "x": qx, "dt": qdt, "B": qB, "C": qC, "A": qA,
+               "in": pg.scan_inputs(qx, qdt, qB, qA, qC, a_kind=pg.PRECOG_A_POWER),
+               "idx": torch.empty(nq, dtype=torch.int64, device=dev),
+               "score": torch.empty(nq, dtype=torch.float32, device=dev),
+               "ws": torch.empty(pg.precog_retrieve_workspace_size(M, dim, nq) + 16,
+                                 dtype=torch.uint8, device=dev),
+               "y": torch.empty((L, nq * Tq, D), dtype=torch.bfloat16, device=dev),
+               "h": torch.empty((nq, L, D, N), dtype=torch.bfloat16, device=dev), "n": nq}
+        return out
+
+    qb = query_batch(Q, seed + 3)
+
+    def query_path(b, stream=None):
+        pg.precog_retrieve(index, b["q"], b["idx"], b["score"], workspace=b["ws"], stream=stream)
+        pg.precog_prefill_from_state(b["in"], b["n"], Tq, qbank, idx=b["idx"], y_out=b["y"],
+                                     state_out=b["h"], stream=stream)
+
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(L * args.steps)]
+
+    def step(k=None):
+        for l in range(L):
+            if k is not None:
+                ev[k * L + l][0].record()
+            pg.precog_encode_chunks(scan_in[l % args.input_sets], off, T, states_out=bank,
+                                    layer0=l, L_total=L)
+            if k is not None:
+                ev[k * L + l][1].record()
+        query_path(qb)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    st, bits = pg.precog_device_status()
+    if st != 0:
+        raise RuntimeError(f"device status {st} bits {bits:#x} after warm-up")
+    ok_rows = bool(torch.equal(qb["idx"], qb["rows"]))
+
+    # ---------------- timed region
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    launches0 = pg.load_library().precog_launch_count()
+    with Clocks(local_rank) as clk:
+        barrier()
+        torch.cuda.synchronize()
+        t0.record()
+        for k in range(args.steps):
+            step(k)
+        t1.record()
+        torch.cuda.synchronize()
+        barrier()
+    launches = pg.load_library().precog_launch_count() - launches0
+    clocks = clk.summary()
+    elapsed_ms = max_over_ranks(t0.elapsed_time(t1))
+    scan_ms = [a.elapsed_time(b) for a, b in ev]
+    tokens_per_step = T
+    value = world * tokens_per_step * args.steps / (elapsed_ms * 1e-3)
+    ms_per_step = elapsed_ms / args.steps
+
+    hbm, peak_src = peaks()
+    bpl = scan_bytes_per_launch(T, shape.n_chunks, D, N)
+    avg_scan_ms = statistics.mean(scan_ms)
+    achieved = bpl / (avg_scan_ms * 1e-3) / 1e9
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                "frac": achieved / hbm, "traffic": profiled_traffic(),
+                "kernel": "scan_kernel (encode, capture)", "peak_source": peak_src,
+                "algorithmic_bytes_per_launch": bpl, "avg_launch_ms": avg_scan_ms}
+
+    # ---------------- query latency (retrieve + inject + prefill), L2 flushed before each
+    latency = {}
+    if not args.no_latency:
+        flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+        for nq, iters in ((1, args.latency_iters), (256, max(20, args.latency_iters // 4))):
+            b = qb if nq == Q else query_batch(nq, seed + 7 + nq)
+            for _ in range(3):
+                query_path(b)
+            times = []
+            for _ in range(iters):
+                flush.zero_()
+                s_ev, e_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                s_ev.record()
+                query_path(b)
+                e_ev.record()
+                e_ev.synchronize()
+                times.append(s_ev.elapsed_time(e_ev) * 1e3)
+            times.sort()
+            latency[f"q{nq}"] = {"p50_us": times[len(times) // 2],
+                                 "p90_us": times[int(len(times) * 0.9)], "iters": iters,
+                                 "retrieved_planted": bool(torch.equal(b["idx"], b["rows"]))}
+            if b is not qb:
+                del b
+        del flush
+
+    # ---------------- end to end: host inputs -> device -> encode/query -> host results
+    e2e = None
+    if not args.no_e2e:
+        host = {k: torch.empty(sets[0][k].shape, dtype=sets[0][k].dtype, pin_memory=True)
+                for k in ("x", "dt", "B")}
+        for k in host:
+            host[k].copy_(sets[0][k])
+        hq = {k: torch.empty(qb[k].shape, dtype=qb[k].dtype, pin_memory=True)
+              for k in ("q", "x", "dt", "B", "C")}
+        for k in hq:
+            hq[k].copy_(qb[k])
+        bank_host = torch.empty(bank.shape, dtype=bank.dtype, pin_memory=True)
+        out_host = {k: torch.empty(qb[k].shape, dtype=qb[k].dtype, pin_memory=True)
+                    for k in ("idx", "score", "y", "h")}
+        copy_stream = torch.cuda.Stream(device=dev)
+        comp = torch.cuda.current_stream(dev)
+        S = args.input_sets
+        h2d = sum(host[k].numel() * host[k].element_size() for k in host) * L
+        h2d += sum(hq[k].numel() * hq[k].element_size() for k in hq)
+        d2h = bank.numel() * bank.element_size()
+        d2h += sum(out_host[k].numel() * out_host[k].element_size() for k in out_host)
+
+        def e2e_step():
+            done = [None] * S              # encode of the layer that last used each buffer
+            copied = []
+            for l in range(L):
+                buf = sets[l % S]
+                with torch.cuda.stream(copy_stream):
+                    if done[l % S] is not None:
+                        copy_stream.wait_event(done[l % S])
+                    for k in ("x", "dt", "B"):
+                        buf[k].copy_(host[k], non_blocking=True)
+                    e = torch.cuda.Event()
+                    e.record(copy_stream)
+                comp.wait_event(e)
+                pg.precog_encode_chunks(scan_in[l % S], off, T, states_out=bank, layer0=l, L_total=L)
+                d = torch.cuda.Event()
+                d.record(comp)
+                done[l % S] = d
+            for k in ("q", "x", "dt", "B", "C"):
+                qb[k].copy_(hq[k], non_blocking=True)
+            query_path(qb)
+            bank_host.copy_(bank, non_blocking=True)
+            for k in out_host:
+                out_host[k].copy_(qb[k], non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize()
+        barrier()
+        w0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            e2e_step()
+        torch.cuda.synchronize()
+        e2e_s = max_over_ranks(time.perf_counter() - w0)
+        barrier()
+        e2e = {"value": world * tokens_per_step * args.e2e_steps / e2e_s, "unit": UNIT,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+               "ms_per_step": 1e3 * e2e_s / args.e2e_steps, "steps": args.e2e_steps}
+        del host, hq, bank_host, out_host
+
+    st, bits = pg.precog_device_status()
+    if st != 0:
+        raise RuntimeError(f"device status {st} bits {bits:#x} after the timed region")
+
+    # ---------------- CPU baseline: the oracle on a bounded sample (rank 0, N=1 only)
+    cpu = None
+    if not args.no_cpu and rank == 0 and world == 1:
+        import oracle
+        chunks = 2
+        xs = sets[0]["x"][: chunks * shape.chunk_len].double().cpu().numpy()
+        dts = sets[0]["dt"][: chunks * shape.chunk_len].double().cpu().numpy()
+        Bs = sets[0]["B"][: chunks * shape.chunk_len].double().cpu().numpy()
+        An = sets[0]["A"].cpu().numpy()
+        offs = synth.fixed_offsets(chunks, shape.chunk_len)
+        oracle.build()
+        c0 = time.perf_counter()
+        oracle.scan(xs, dts, An, Bs, offs)
+        c_s = time.perf_counter() - c0
+        cpu = {"value": chunks * shape.chunk_len / c_s / L, "unit": UNIT, "cores": 1,
+               "kind": "oracle",
+               "sample": f"{chunks} chunks x {shape.chunk_len} tokens x 1 layer of this workload "
+                         f"(fp64 sequential oracle, one core), rate divided by {L} layers",
+               "seconds": c_s}
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": "f32", "io_dtype": "bf16", "data": "synthetic",
+                "config": {"workload": "paper-shaped corpus encode + query-time path",
+                           "layers": L, "D": D, "N": N, "chunks": shape.n_chunks,
+                           "chunk_tokens": shape.chunk_len, "state_bytes_per_chunk": L * D * N * 2,
+                           "input_sets_resident": args.input_sets,
+                           "index_rows": M, "index_dim": dim, "bank_entries": M,
+                           "query_batch": Q, "query_tokens": Tq, "parallelism": f"dp{world}",
+                           "l2": "inputs larger than L2 (12.98 GB per layer, 1.5 GB index)"},
+                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks,
+                "gpu_launches": int(launches), "latency": latency,
+                "retrieved_planted": ok_rows, "input_gen_s_per_layer": gen_s_per_layer}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -51,10 +51,17 @@ typedef enum precog_dtype {
     PRECOG_F16 = 2
 } precog_dtype;
 
+/* Structure of the diagonal state matrix A (see precog_scan_inputs). */
+typedef enum precog_a_kind {
+    PRECOG_A_GENERAL = 0,  /* any A: one exponential per (channel, state index) */
+    PRECOG_A_POWER = 1     /* A[d,n] == (n+1)*A[d,0] exactly and A[d,0] <= 0 */
+} precog_a_kind;
+
 /* Device status bits reported by precog_device_status(). */
 #define PRECOG_DEV_BAD_OFFSETS 0x1u  /* offsets not non-decreasing or beyond T_tot */
 #define PRECOG_DEV_BAD_INDEX 0x2u    /* a bank row index outside [-1, bank_entries) */
 #define PRECOG_DEV_TIMEOUT 0x4u      /* an mbarrier wait hit its iteration limit */
+#define PRECOG_DEV_BAD_A 0x8u        /* a_kind == PRECOG_A_POWER but A is not */
 
 /*
  * Inputs of the selective-SSM scan for L layers (Sec. 3, Eq. 1).
@@ -76,15 +83,21 @@ typedef enum precog_dtype {
  * layer block 16-byte aligned; they may be 0 when n_layers == 1.
  * Requirements: N == 16; D >= 1 with D*sizeof(in_dtype) a multiple of 16.
  * x, dt and B (and C) may be NULL only when there are no token rows.
- * When A[d,n] == (n+1)*A[d,0] holds exactly for every n of a channel group,
- * the kernel derives alpha_n as a power of one exponential (the same value
- * up to fp32 rounding); otherwise it takes one exponential per (d, n).
+ *
+ * a_kind selects the update form. PRECOG_A_GENERAL accepts any A and takes
+ * one exponential per (d, n). PRECOG_A_POWER is the caller's statement that
+ * A[d,n] == (n+1)*A[d,0] exactly with A[d,0] <= 0 (e.g. A[d,n] = -(n+1)), so
+ * that alpha_n = r^(n+1) with r = exp(dt*A[d,0]): one exponential per (t, d).
+ * The kernel verifies the statement per block of channels; where it is false
+ * nothing is written for that block and PRECOG_DEV_BAD_A is flagged.
  */
 typedef struct precog_scan_inputs {
     int32_t n_layers;
     int32_t D;
     int32_t N;
     int32_t in_dtype;          /* precog_dtype */
+    int32_t a_kind;            /* precog_a_kind */
+    int32_t reserved;          /* must be 0 */
     const void *x;
     const void *dt;
     const void *B;
@@ -190,6 +203,10 @@ const char *precog_last_error(void);
 
 /* PRECOG_ABI_VERSION of the loaded library. */
 int32_t precog_abi_version(void);
+
+/* Number of CUDA kernels this library has launched in this process (all
+ * devices, all threads); callers difference it around a region of work. */
+uint64_t precog_launch_count(void);
 
 #ifdef __cplusplus
 }

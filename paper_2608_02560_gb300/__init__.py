@@ -23,7 +23,8 @@ LIB_PATH = os.path.join(_PKG, "libprecog.so")
 
 PRECOG_F32, PRECOG_BF16, PRECOG_F16 = 0, 1, 2
 PRECOG_OK = 0
-PRECOG_DEV_BAD_OFFSETS, PRECOG_DEV_BAD_INDEX, PRECOG_DEV_TIMEOUT = 0x1, 0x2, 0x4
+PRECOG_A_GENERAL, PRECOG_A_POWER = 0, 1
+PRECOG_DEV_BAD_OFFSETS, PRECOG_DEV_BAD_INDEX, PRECOG_DEV_TIMEOUT, PRECOG_DEV_BAD_A = 0x1, 0x2, 0x4, 0x8
 STATUS_NAMES = {0: "PRECOG_OK", 1: "PRECOG_ERR_INVALID_ARG", 2: "PRECOG_ERR_UNSUPPORTED",
                 3: "PRECOG_ERR_CUDA", 4: "PRECOG_ERR_TIMEOUT", 5: "PRECOG_ERR_DEVICE"}
 
@@ -38,7 +39,8 @@ class PrecogError(RuntimeError):
 class ScanInputs(ctypes.Structure):
     """Mirror of ``precog_scan_inputs`` (include/precog.h)."""
     _fields_ = [("n_layers", ctypes.c_int32), ("D", ctypes.c_int32), ("N", ctypes.c_int32),
-                ("in_dtype", ctypes.c_int32), ("x", ctypes.c_void_p), ("dt", ctypes.c_void_p),
+                ("in_dtype", ctypes.c_int32), ("a_kind", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("x", ctypes.c_void_p), ("dt", ctypes.c_void_p),
                 ("B", ctypes.c_void_p), ("C", ctypes.c_void_p), ("A", ctypes.c_void_p),
                 ("layer_stride_xd", ctypes.c_int64), ("layer_stride_bc", ctypes.c_int64)]
 
@@ -111,8 +113,11 @@ def _stream(stream):
     return ctypes.c_void_p(stream.cuda_stream)
 
 
-def scan_inputs(x, dt, B, A, C=None) -> ScanInputs:
-    """Describe x, dt ``[L, T, D]`` (or ``[T, D]``), B, C ``[L, T, N]``, A ``[L, D, N]``."""
+def scan_inputs(x, dt, B, A, C=None, a_kind: int = PRECOG_A_GENERAL) -> ScanInputs:
+    """Describe x, dt ``[L, T, D]`` (or ``[T, D]``), B, C ``[L, T, N]``, A ``[L, D, N]``.
+
+    ``a_kind=PRECOG_A_POWER`` states that A[d, n] == (n + 1) * A[d, 0] <= 0 (verified on
+    the device); it selects the one-exponential update forms."""
     if x.dim() == 2:
         x, dt, B = x.unsqueeze(0), dt.unsqueeze(0), B.unsqueeze(0)
         C = None if C is None else C.unsqueeze(0)
@@ -128,6 +133,7 @@ def scan_inputs(x, dt, B, A, C=None) -> ScanInputs:
     s = ScanInputs()
     s.n_layers, s.D, s.N = L, D, N
     s.in_dtype = _dtype_code(x)
+    s.a_kind = a_kind
     s.x, s.dt, s.B, s.C, s.A = _ptr(x), _ptr(dt), _ptr(B), _ptr(C), _ptr(A)
     s.layer_stride_xd = T * D
     s.layer_stride_bc = T * N

@@ -1,6 +1,8 @@
 // C ABI of the PRECOG hot path: argument validation, dispatch to the
 // kernels, status codes. Nothing here allocates device memory.
+#include <atomic>
 #include <cstdarg>
+#include <mutex>
 #include <cstdio>
 #include <cstring>
 
@@ -47,6 +49,8 @@ precog_status check_scan_inputs(const precog_scan_inputs *in, int64_t rows, bool
     if (in->n_layers < 1) return fail(PRECOG_ERR_INVALID_ARG, "n_layers must be >= 1");
     if (in->N != 16) return fail(PRECOG_ERR_UNSUPPORTED, "N=%d: only N=16 is implemented", in->N);
     if (in->D < 1) return fail(PRECOG_ERR_INVALID_ARG, "D must be >= 1");
+    if (in->a_kind != PRECOG_A_GENERAL && in->a_kind != PRECOG_A_POWER)
+        return fail(PRECOG_ERR_INVALID_ARG, "a_kind must be PRECOG_A_GENERAL or PRECOG_A_POWER");
     if (in->in_dtype != PRECOG_F32 && in->in_dtype != PRECOG_BF16)
         return fail(PRECOG_ERR_UNSUPPORTED, "in_dtype must be PRECOG_F32 or PRECOG_BF16");
     const int sz = dtype_size(in->in_dtype);
@@ -83,11 +87,29 @@ precog::ScanParams base_params(const precog_scan_inputs *in, int64_t rows) {
     p.D = in->D;
     p.N = in->N;
     p.in_dtype = in->in_dtype;
+    p.a_kind = in->a_kind;
     p.T_tot = rows;
     return p;
 }
 
+std::atomic<uint64_t> g_launches{0};
+std::mutex g_attr_mutex;
+
 }  // namespace
+
+namespace precog {
+
+void count_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+
+cudaError_t ensure_smem(const void *kernel, int *cached_bytes, int bytes) {
+    std::lock_guard<std::mutex> lock(g_attr_mutex);
+    if (*cached_bytes >= bytes) return cudaSuccess;
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess) *cached_bytes = bytes;
+    return e;
+}
+
+}  // namespace precog
 
 extern "C" {
 
@@ -190,7 +212,8 @@ precog_status precog_retrieve(const void *index, int32_t index_dtype, int64_t M,
     if (dim < 1) return fail(PRECOG_ERR_INVALID_ARG, "dim must be >= 1");
     if ((static_cast<int64_t>(dim) * sz) % 16 != 0)
         return fail(PRECOG_ERR_UNSUPPORTED, "dim*sizeof(dtype) must be a multiple of 16");
-    if (dim > 4096) return fail(PRECOG_ERR_UNSUPPORTED, "dim > 4096 is not implemented");
+    if (static_cast<int64_t>(dim) * sz > 8192)
+        return fail(PRECOG_ERR_UNSUPPORTED, "rows longer than 8 KiB (dim*sizeof(dtype)) are not implemented");
     if (n_queries < 0) return fail(PRECOG_ERR_INVALID_ARG, "n_queries must be >= 0");
     if (n_queries == 0) return ok();
     if ((M > 0 && index == nullptr) || queries == nullptr || d_best_idx == nullptr)
@@ -230,7 +253,7 @@ precog_status precog_device_status(void *stream, uint32_t *bits_out) {
     if (*bits_out == 0) return ok();
     if (*bits_out & PRECOG_DEV_TIMEOUT)
         return fail(PRECOG_ERR_TIMEOUT, "a device-side wait gave up (bits 0x%x)", *bits_out);
-    return fail(PRECOG_ERR_DEVICE, "device flagged invalid offsets or bank rows (bits 0x%x)", *bits_out);
+    return fail(PRECOG_ERR_DEVICE, "device flagged invalid offsets, bank rows or A (bits 0x%x)", *bits_out);
 }
 
 const char *precog_status_string(int32_t status) {
@@ -248,5 +271,7 @@ const char *precog_status_string(int32_t status) {
 const char *precog_last_error(void) { return g_last_error; }
 
 int32_t precog_abi_version(void) { return PRECOG_ABI_VERSION; }
+
+uint64_t precog_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
 }  // extern "C"

@@ -16,6 +16,7 @@ struct ScanParams {
     int64_t ls_xd, ls_bc;     // layer strides in elements
     int32_t n_layers, D, N;
     int32_t in_dtype;         // precog_dtype
+    int32_t a_kind;           // precog_a_kind
     int64_t T_tot;            // rows per layer
     // chunking: use_fixed -> chunk c is rows [c*fixed_len, (c+1)*fixed_len),
     // else rows [offsets[c], offsets[c+1])
@@ -37,6 +38,13 @@ struct ScanParams {
     void *y;                  // [L][T_tot][D] or nullptr
     int32_t y_dtype;
 };
+
+// Kernel launches made by this library since the process started.
+void count_launches(uint64_t n);
+
+// Raise a kernel's dynamic shared-memory limit once per process (a host-side
+// attribute, not a stream operation, so later calls stay graph-capturable).
+cudaError_t ensure_smem(const void *kernel, int *cached_bytes, int bytes);
 
 cudaError_t launch_scan(const ScanParams &p, cudaStream_t stream);
 cudaError_t scan_status_word_read_clear(uint32_t *bits);

@@ -2,9 +2,9 @@
 //
 // Batched GEMV on the CUDA cores: every warp streams whole key rows with
 // 16-byte loads (several rows in flight per warp), dots them with a group of
-// up to kQB queries held in shared memory as fp32, and reduces across lanes
-// with a fixed butterfly, so a row's score never depends on where the row
-// sits: equal rows get equal scores and the lowest row wins a tie. Each
+// up to kQB queries held in registers as fp32, and reduces across lanes with
+// a fixed butterfly, so a row's score never depends on where the row sits:
+// equal rows get equal scores and the lowest row wins a tie. Each
 // (score, row) pair is packed into one 64-bit key ordered by score, then by
 // lower row; per-CTA maxima go to the workspace and a finalize kernel reduces
 // them. A NaN score never enters a key, so it never wins.
@@ -22,8 +22,7 @@ __device__ uint32_t g_retrieve_status;
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int kQB = 4;        // queries per pass over the index
-constexpr int kRowsInFlight = 4;
-constexpr int kMaxDim = 4096;
+constexpr int kMaxVecsPerRow = 512;  // 16 vectors per lane
 
 // Monotone map of a non-NaN fp32 score to uint32 (-inf -> 0x007fffff > 0).
 __device__ __forceinline__ uint32_t ordered_bits(float s) {
@@ -69,70 +68,77 @@ __device__ __forceinline__ void widen(const uint4 &v, float (&f)[Vec<T>::n]) {
 }
 
 // partial[blockIdx.x * n_queries + q] = best key of this CTA for query q.
-template <typename T>
+// Lane l owns the 16-byte vectors l, l+32, ... of every row (VPL of them) and
+// holds the matching query values in registers; RIF rows are loaded before any
+// is used, so each lane keeps RIF*VPL 16-byte loads in flight.
+template <typename T, int QB, int VPL, int RIF>
 __global__ void __launch_bounds__(kThreads)
     gemv_top1_kernel(const T *__restrict__ index, int64_t M, int dim, const T *__restrict__ queries,
                      int n_queries, int q0, unsigned long long *__restrict__ partial) {
     constexpr int V = Vec<T>::n;
-    extern __shared__ float qs[];  // [kQB][dim]
-    __shared__ unsigned long long best[kQB];
-    const int nq = min(kQB, n_queries - q0);
-    for (int i = threadIdx.x; i < kQB * dim; i += kThreads) {
-        const int qq = i / dim, k = i % dim;
-        qs[i] = (qq < nq) ? to_f32(queries[static_cast<int64_t>(q0 + qq) * dim + k]) : 0.f;
-    }
-    if (threadIdx.x < kQB) best[threadIdx.x] = 0ull;
-    __syncthreads();
-
+    __shared__ unsigned long long best[QB];
+    const int nq = min(QB, n_queries - q0);
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
-    const int64_t gwarp = static_cast<int64_t>(blockIdx.x) * kWarps + warp;
-    const int64_t nwarps = static_cast<int64_t>(gridDim.x) * kWarps;
-    const int vecs = dim / V;              // 16-byte vectors per row
-    unsigned long long mykey[kQB];
+    const int vecs = dim / V;
+    float qv[QB][VPL][V];
 #pragma unroll
-    for (int qq = 0; qq < kQB; ++qq) mykey[qq] = 0ull;
-
-    for (int64_t r0 = gwarp * kRowsInFlight; r0 < M; r0 += nwarps * kRowsInFlight) {
-        float acc[kRowsInFlight][kQB];
+    for (int qq = 0; qq < QB; ++qq)
 #pragma unroll
-        for (int r = 0; r < kRowsInFlight; ++r)
+        for (int j = 0; j < VPL; ++j) {
+            const int v = lane + 32 * j;
+            if (qq < nq && v < vecs) {
+                const uint4 raw =
+                    __ldg(reinterpret_cast<const uint4 *>(queries + static_cast<int64_t>(q0 + qq) * dim) + v);
+                widen<T>(raw, qv[qq][j]);
+            } else {
 #pragma unroll
-            for (int qq = 0; qq < kQB; ++qq) acc[r][qq] = 0.f;
-        for (int v0 = 0; v0 < vecs; v0 += 32) {
-            const int v = v0 + lane;
-            uint4 raw[kRowsInFlight];
-#pragma unroll
-            for (int r = 0; r < kRowsInFlight; ++r) {
-                const int64_t row = r0 + r;
-                raw[r] = (v < vecs && row < M)
-                             ? __ldg(reinterpret_cast<const uint4 *>(index + row * dim) + v)
-                             : make_uint4(0, 0, 0, 0);
-            }
-            if (v < vecs) {
-#pragma unroll
-                for (int r = 0; r < kRowsInFlight; ++r) {
-                    float f[V];
-                    widen<T>(raw[r], f);
-#pragma unroll
-                    for (int qq = 0; qq < kQB; ++qq) {
-                        const float *qv = qs + qq * dim + v * V;
-#pragma unroll
-                        for (int e = 0; e < V; ++e) acc[r][qq] = fmaf(f[e], qv[e], acc[r][qq]);
-                    }
-                }
+                for (int e = 0; e < V; ++e) qv[qq][j][e] = 0.f;
             }
         }
+    if (threadIdx.x < QB) best[threadIdx.x] = 0ull;
+    __syncthreads();
+
+    const int64_t gwarp = static_cast<int64_t>(blockIdx.x) * kWarps + warp;
+    const int64_t nwarps = static_cast<int64_t>(gridDim.x) * kWarps;
+    unsigned long long mykey[QB];
 #pragma unroll
-        for (int r = 0; r < kRowsInFlight; ++r) {
+    for (int qq = 0; qq < QB; ++qq) mykey[qq] = 0ull;
+
+    for (int64_t r0 = gwarp * RIF; r0 < M; r0 += nwarps * RIF) {
+        uint4 raw[RIF][VPL];
 #pragma unroll
-            for (int qq = 0; qq < kQB; ++qq) {
-                float s = acc[r][qq];
+        for (int r = 0; r < RIF; ++r)
 #pragma unroll
-                for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+            for (int j = 0; j < VPL; ++j) {
+                const int v = lane + 32 * j;
                 const int64_t row = r0 + r;
-                if (row < M && !isnan(s)) {
-                    const unsigned long long key = make_key(s, row);
+                raw[r][j] = (v < vecs && row < M)
+                                ? __ldg(reinterpret_cast<const uint4 *>(index + row * dim) + v)
+                                : make_uint4(0, 0, 0, 0);
+            }
+#pragma unroll
+        for (int r = 0; r < RIF; ++r) {
+            float acc[QB];
+#pragma unroll
+            for (int qq = 0; qq < QB; ++qq) acc[qq] = 0.f;
+#pragma unroll
+            for (int j = 0; j < VPL; ++j) {
+                float f[V];
+                widen<T>(raw[r][j], f);
+#pragma unroll
+                for (int qq = 0; qq < QB; ++qq)
+#pragma unroll
+                    for (int e = 0; e < V; ++e) acc[qq] = fmaf(f[e], qv[qq][j][e], acc[qq]);
+            }
+            const int64_t row = r0 + r;
+#pragma unroll
+            for (int qq = 0; qq < QB; ++qq) {
+                float sc = acc[qq];
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) sc += __shfl_xor_sync(0xffffffffu, sc, o);
+                if (row < M && !isnan(sc)) {
+                    const unsigned long long key = make_key(sc, row);
                     mykey[qq] = key > mykey[qq] ? key : mykey[qq];
                 }
             }
@@ -175,32 +181,55 @@ int num_sms() {
     return sms;
 }
 
+constexpr int kRowsPerWarpPass = 4;
+
 int gemv_grid(int64_t M) {
-    const int64_t rows_per_cta = static_cast<int64_t>(kWarps) * kRowsInFlight;
+    const int64_t rows_per_cta = static_cast<int64_t>(kWarps) * kRowsPerWarpPass;
     const int64_t need = (M + rows_per_cta - 1) / rows_per_cta;
     const int64_t cap = static_cast<int64_t>(num_sms()) * 4;
     return static_cast<int>(need < 1 ? 1 : (need < cap ? need : cap));
 }
 
+template <typename T, int QB, int VPL>
+cudaError_t launch_gemv_pass(const RetrieveParams &p, int grid, int q0, cudaStream_t stream) {
+    constexpr int RIF = QB == 1 ? 4 : 2;
+    gemv_top1_kernel<T, QB, VPL, RIF><<<grid, kThreads, 0, stream>>>(
+        static_cast<const T *>(p.index), p.M, p.dim, static_cast<const T *>(p.queries), p.n_queries,
+        q0, static_cast<unsigned long long *>(p.workspace));
+    return cudaGetLastError();
+}
+
+template <typename T, int QB>
+cudaError_t gemv_pass_vpl(const RetrieveParams &p, int grid, int q0, cudaStream_t stream) {
+    const int vecs = p.dim / Vec<T>::n;
+    const int vpl = (vecs + 31) / 32;
+    if (vpl <= 1) return launch_gemv_pass<T, QB, 1>(p, grid, q0, stream);
+    if (vpl <= 2) return launch_gemv_pass<T, QB, 2>(p, grid, q0, stream);
+    if (vpl <= 3) return launch_gemv_pass<T, QB, 3>(p, grid, q0, stream);
+    if (vpl <= 4) return launch_gemv_pass<T, QB, 4>(p, grid, q0, stream);
+    if (vpl <= 8) return launch_gemv_pass<T, QB, 8>(p, grid, q0, stream);
+    return launch_gemv_pass<T, QB, 16>(p, grid, q0, stream);
+}
+
 template <typename T>
 cudaError_t launch_gemv(const RetrieveParams &p, cudaStream_t stream) {
     const int grid = gemv_grid(p.M);
-    const size_t smem = static_cast<size_t>(kQB) * p.dim * sizeof(float);
-    auto kern = gemv_top1_kernel<T>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
-    if (e != cudaSuccess) return e;
     auto *partial = static_cast<unsigned long long *>(p.workspace);
-    for (int q0 = 0; q0 < p.n_queries; q0 += kQB) {
-        kern<<<grid, kThreads, smem, stream>>>(static_cast<const T *>(p.index), p.M, p.dim,
-                                               static_cast<const T *>(p.queries), p.n_queries, q0,
-                                               partial);
-        e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
+    uint64_t launches = 0;
+    cudaError_t e = cudaSuccess;
+    if (p.n_queries == 1) {
+        e = gemv_pass_vpl<T, 1>(p, grid, 0, stream);
+        ++launches;
+    } else {
+        for (int q0 = 0; q0 < p.n_queries && e == cudaSuccess; q0 += kQB, ++launches)
+            e = gemv_pass_vpl<T, kQB>(p, grid, q0, stream);
     }
+    if (e != cudaSuccess) return e;
     finalize_kernel<<<(p.n_queries + 127) / 128, 128, 0, stream>>>(partial, grid, p.n_queries,
                                                                     p.best_idx, p.best_score);
-    return cudaGetLastError();
+    e = cudaGetLastError();
+    if (e == cudaSuccess) count_launches(launches + 1);
+    return e;
 }
 
 }  // namespace
@@ -213,7 +242,8 @@ size_t retrieve_workspace_size(int64_t M, int32_t dim, int32_t n_queries) {
 
 cudaError_t launch_retrieve(const RetrieveParams &p, cudaStream_t stream) {
     if (p.n_queries == 0) return cudaSuccess;
-    if (p.dim > kMaxDim) return cudaErrorInvalidValue;
+    const int sz = p.dtype == PRECOG_F32 ? 4 : 2;
+    if (p.dim * sz / 16 > kMaxVecsPerRow) return cudaErrorInvalidValue;
     switch (p.dtype) {
         case PRECOG_F16: return launch_gemv<__half>(p, stream);
         case PRECOG_BF16: return launch_gemv<__nv_bfloat16>(p, stream);

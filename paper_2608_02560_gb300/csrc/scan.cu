@@ -200,12 +200,182 @@ __device__ __forceinline__ void scan_tile(const unsigned char *st, const StageLa
     }
 }
 
-template <typename TIn, bool HAS_Y, bool HAS_H0>
-__global__ void __launch_bounds__(kMaxThreads, 3)
+// ---------------------------------------------------------------------------
+// Rescaled accumulation (capture without readout, A[d, n] = (n + 1) * a, a <= 0).
+// With E_t = 2^(L_t), L_t = sum over the tokens since the last renormalisation
+// of dt * (-a * log2 e), the state is h_n = E_t^-(n+1) * G_n and one token adds
+//   G_n += (u * E_t^(n+1)) * B_n,     u = dt * x,
+// so the per-n decay multiply of the direct update disappears: per token and
+// channel one exponential, a packed power chain and 16 FMAs. Whenever some
+// lane's L would pass kLmax the whole warp renormalises (h_n = G_n E^-(n+1),
+// L = 0), which keeps E^16 <= 2^(16 * kLmax) far from fp32 overflow. A single
+// token whose own increment exceeds kLmax is applied directly to h.
+constexpr float kLmax = 6.0f;
+
+// p[i] = (r^(2i+1), r^(2i+2)) for i = 0..7
+__device__ __forceinline__ void pow_pairs(float r, f2 (&p)[8]) {
+    const float r2 = r * r;
+    p[0] = pack2(r, r2);
+    const f2 rr = pack2(r2, r2);
+#pragma unroll
+    for (int i = 1; i < 8; ++i) p[i] = mul2(p[i - 1], rr);
+}
+
+__device__ __forceinline__ void renormalise(f2 (&g)[8], float &L) {
+    f2 p[8];
+    pow_pairs(ex2(-L), p);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) g[i] = mul2(g[i], p[i]);
+    L = 0.f;
+}
+
+// G_n += u * 2^((n+1) * Ln) * B_n
+__device__ __forceinline__ void accumulate(f2 (&g)[8], const f2 (&b)[8], float u, float Ln) {
+    const float E = ex2(Ln);
+    const float w0 = u * E;
+    const float E2 = E * E;
+    f2 w = pack2(w0, w0 * E);
+    const f2 ee = pack2(E2, E2);
+    g[0] = fma2(w, b[0], g[0]);
+#pragma unroll
+    for (int i = 1; i < 8; ++i) {
+        w = mul2(w, ee);
+        g[i] = fma2(w, b[i], g[i]);
+    }
+}
+
+// One token with the window check: renormalise the whole warp when some lane
+// would leave [-kLmax, kLmax]; a token whose own increment is outside it is
+// applied to h directly (alpha_n = 2^(-(n+1)*Ln)) and contributes nothing to G.
+__device__ __forceinline__ void token_checked(f2 (&g)[kCPT][8], float (&L)[kCPT],
+                                              const float (&kk)[kCPT], const f2 (&b)[8],
+                                              const float (&xv)[kCPT], const float (&dv)[kCPT],
+                                              unsigned wmask) {
+    float Ln[kCPT], u[kCPT];
+    bool need = false;
+#pragma unroll
+    for (int j = 0; j < kCPT; ++j) {
+        Ln[j] = fmaf(dv[j], kk[j], L[j]);
+        u[j] = dv[j] * xv[j];
+        need |= !(fabsf(Ln[j]) <= kLmax);
+    }
+    if (__any_sync(wmask, need)) {
+#pragma unroll
+        for (int j = 0; j < kCPT; ++j) {
+            renormalise(g[j], L[j]);
+            Ln[j] = dv[j] * kk[j];
+            if (!(fabsf(Ln[j]) <= kLmax)) {
+                f2 a[8];
+                pow_pairs(ex2(-Ln[j]), a);
+                const f2 uu = pack2(u[j], u[j]);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) g[j][i] = fma2(a[i], g[j][i], mul2(uu, b[i]));
+                Ln[j] = 0.f;
+                u[j] = 0.f;
+            }
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < kCPT; ++j) {
+        accumulate(g[j], b, u[j], Ln[j]);
+        L[j] = Ln[j];
+    }
+}
+
+template <typename TIn>
+__device__ __forceinline__ void load_token(const unsigned char *st, const StageLayout &lay,
+                                           const float *bsrc, int DS, int dl, int t, f2 (&b)[8],
+                                           float (&xv)[kCPT], float (&dv)[kCPT]) {
+    constexpr int sz = sizeof(TIn);
+    const ulonglong2 *bv = reinterpret_cast<const ulonglong2 *>(bsrc + t * kN);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const ulonglong2 v = bv[i];
+        b[2 * i] = v.x;
+        b[2 * i + 1] = v.y;
+    }
+    load_pair<TIn>(st + lay.xs + (t * DS + dl) * sz, xv[0], xv[1]);
+    load_pair<TIn>(st + lay.dts + (t * DS + dl) * sz, dv[0], dv[1]);
+}
+
+// Tokens go in groups of kGroup: the exponents of the whole group are summed
+// first (one serial FMA per token), one warp vote decides whether the group
+// stays inside the window, and then the group's accumulations carry no branch,
+// so the scheduler can interleave the power chains of its tokens.
+constexpr int kGroup = 4;
+
+template <typename TIn>
+__device__ __forceinline__ void scan_tile_rescaled(const unsigned char *st, const StageLayout &lay,
+                                                   int DS, int dl, int ntok, f2 (&g)[kCPT][8],
+                                                   float (&L)[kCPT], const float (&kk)[kCPT],
+                                                   unsigned wmask) {
+    constexpr bool CONV = !std::is_same<TIn, float>::value;
+    constexpr int sz = sizeof(TIn);
+    const float *bsrc = reinterpret_cast<const float *>(st + (CONV ? lay.bf : lay.bs));
+    int t = 0;
+    for (; t + kGroup <= ntok; t += kGroup) {
+        float Lk[kGroup][kCPT];
+        bool need = false;
+#pragma unroll
+        for (int k = 0; k < kGroup; ++k) {
+            float dv[kCPT], xv[kCPT];
+            load_pair<TIn>(st + lay.dts + ((t + k) * DS + dl) * sz, dv[0], dv[1]);
+#pragma unroll
+            for (int j = 0; j < kCPT; ++j) {
+                Lk[k][j] = fmaf(dv[j], kk[j], k ? Lk[k - 1][j] : L[j]);
+                need |= !(fabsf(Lk[k][j]) <= kLmax);
+            }
+            (void)xv;
+        }
+        if (__any_sync(wmask, need)) {
+#pragma unroll 1
+            for (int k = 0; k < kGroup; ++k) {
+                f2 b[8];
+                float xv[kCPT], dv[kCPT];
+                load_token<TIn>(st, lay, bsrc, DS, dl, t + k, b, xv, dv);
+                token_checked(g, L, kk, b, xv, dv, wmask);
+            }
+        } else {
+#pragma unroll
+            for (int k = 0; k < kGroup; ++k) {
+                f2 b[8];
+                float xv[kCPT], dv[kCPT];
+                load_token<TIn>(st, lay, bsrc, DS, dl, t + k, b, xv, dv);
+#pragma unroll
+                for (int j = 0; j < kCPT; ++j) accumulate(g[j], b, dv[j] * xv[j], Lk[k][j]);
+            }
+#pragma unroll
+            for (int j = 0; j < kCPT; ++j) L[j] = Lk[kGroup - 1][j];
+        }
+    }
+    for (; t < ntok; ++t) {
+        f2 b[8];
+        float xv[kCPT], dv[kCPT];
+        load_token<TIn>(st, lay, bsrc, DS, dl, t, b, xv, dv);
+        token_checked(g, L, kk, b, xv, dv, wmask);
+    }
+}
+
+// Update form of one kernel instantiation. kGeneral: one exponential per
+// (d, n). kPower: A[d, n] = (n + 1) * A[d, 0] (the caller states it, every CTA
+// verifies it): with readout, the direct update with a packed power chain;
+// without readout, the rescaled accumulation above.
+enum Mode { kGeneral = 0, kPower = 1 };
+
+template <int MODE, bool HAS_Y> struct Shape {
+    static constexpr bool kRescaled = MODE == kPower && !HAS_Y;
+    static constexpr int kStagesUsed = kRescaled ? 2 : kStages;
+    static constexpr int kMinBlocks = kRescaled ? 4 : 3;
+};
+
+template <typename TIn, bool HAS_Y, bool HAS_H0, int MODE>
+__global__ void __launch_bounds__(kMaxThreads, (Shape<MODE, HAS_Y>::kMinBlocks))
     scan_kernel(const ScanParams p, const int DS, const int slices) {
     extern __shared__ __align__(128) unsigned char smem[];
     constexpr int sz = sizeof(TIn);
     constexpr bool CONV = !std::is_same<TIn, float>::value;
+    constexpr bool RESCALED = Shape<MODE, HAS_Y>::kRescaled;
+    constexpr int STAGES = Shape<MODE, HAS_Y>::kStagesUsed;
     uint64_t *full = reinterpret_cast<uint64_t *>(smem);
     unsigned char *stage0 = smem + kBarBytes;
     const StageLayout lay = stage_layout(DS, sz, HAS_Y, CONV);
@@ -240,15 +410,43 @@ __global__ void __launch_bounds__(kMaxThreads, 3)
     const TIn *Cl = HAS_Y ? static_cast<const TIn *>(p.C) + layer * p.ls_bc : nullptr;
     const float *Al = p.A + static_cast<int64_t>(layer) * D * kN;
 
-    // ---- pipeline start: barrier init, first kStages tiles in flight ----
+    // ---- coefficients; kPower verifies the structure before any copy is issued ----
+    float kpow[kCPT];                      // A[d, 0] * log2 e
+    f2 kgen[kCPT][8];                      // (A[d, n] * log2 e) pairs, kGeneral only
+#pragma unroll
+    for (int j = 0; j < kCPT; ++j) {
+        const float *a = Al + static_cast<int64_t>(d0 + dl + j) * kN;
+        kpow[j] = a[0] * kLog2e;
+        if constexpr (MODE == kGeneral) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) kgen[j][i] = pack2(a[2 * i] * kLog2e, a[2 * i + 1] * kLog2e);
+        }
+    }
+    if constexpr (MODE == kPower) {
+        bool ok = true;
+#pragma unroll
+        for (int j = 0; j < kCPT; ++j) {
+            const float *a = Al + static_cast<int64_t>(d0 + dl + j) * kN;
+            const float a0 = a[0];
+            ok &= a0 <= 0.f;
+#pragma unroll
+            for (int n = 1; n < kN; ++n) ok &= a[n] == static_cast<float>(n + 1) * a0;
+        }
+        if (!__syncthreads_and(ok)) {
+            if (tid == 0) atomicOr(&g_scan_status, PRECOG_DEV_BAD_A);
+            return;
+        }
+    }
+
+    // ---- pipeline start: barrier init, first STAGES tiles in flight ----
     const int64_t ntiles = (len + kTile - 1) / kTile;
     if (tid == 0) {
-        for (int s = 0; s < kStages; ++s) mbar_init(&full[s], 1);
+        for (int s = 0; s < STAGES; ++s) mbar_init(&full[s], 1);
         fence_barrier_init();
     }
     __syncthreads();
     auto issue = [&](int64_t k) {  // thread 0 only
-        const int s = static_cast<int>(k % kStages);
+        const int s = static_cast<int>(k % STAGES);
         unsigned char *st = stage0 + s * lay.bytes;
         const int64_t row0 = start + k * kTile;
         const int ntok = static_cast<int>(min64(kTile, len - k * kTile));
@@ -268,27 +466,9 @@ __global__ void __launch_bounds__(kMaxThreads, 3)
         if (HAS_Y) bulk_g2s(st + lay.cs, Cl + row0 * kN, ntok * kN * sz, &full[s]);
     };
     if (tid == 0)
-        for (int64_t k = 0; k < min64(kStages, ntiles); ++k) issue(k);
+        for (int64_t k = 0; k < min64(STAGES, ntiles); ++k) issue(k);
 
-    // ---- coefficients and the A-structure check (overlaps the first copies) ----
-    float kpow[kCPT];
-    f2 kgen[kCPT][8];
-    bool pow_ok = true;
-#pragma unroll
-    for (int j = 0; j < kCPT; ++j) {
-        const float *a = Al + static_cast<int64_t>(d0 + dl + j) * kN;
-        const float a0 = a[0];
-        kpow[j] = a0 * kLog2e;
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            const float an0 = a[2 * i], an1 = a[2 * i + 1];
-            pow_ok &= (an0 == static_cast<float>(2 * i + 1) * a0) &&
-                      (an1 == static_cast<float>(2 * i + 2) * a0);
-            kgen[j][i] = pack2(an0 * kLog2e, an1 * kLog2e);
-        }
-    }
-
-    // ---- initial state ----
+    // ---- initial state (overlaps the first copies) ----
     f2 h[kCPT][8];
     bool h0_valid = false;
     int64_t h0_row = 0;
@@ -309,19 +489,25 @@ __global__ void __launch_bounds__(kMaxThreads, 3)
             for (int i = 0; i < 8; ++i) h[j][i] = 0;
         }
     }
-    const bool use_pow = __syncthreads_and(pow_ok);
+    const unsigned wmask = __activemask();
+    float Lw[kCPT], kk[kCPT];
+#pragma unroll
+    for (int j = 0; j < kCPT; ++j) {
+        Lw[j] = 0.f;
+        kk[j] = -kpow[j];
+    }
 
     // ---- time loop ----
     void *yrow = nullptr;
-    int64_t y_stride = D;
+    const int64_t y_stride = D;
     if (HAS_Y) {
         const int64_t off = (static_cast<int64_t>(layer) * p.T_tot + start) * D + d0 + dl;
         yrow = (p.y_dtype == PRECOG_F32) ? static_cast<void *>(static_cast<float *>(p.y) + off)
                                          : static_cast<void *>(static_cast<__nv_bfloat16 *>(p.y) + off);
     }
     for (int64_t k = 0; k < ntiles; ++k) {
-        const int s = static_cast<int>(k % kStages);
-        const uint32_t par = static_cast<uint32_t>((k / kStages) & 1);
+        const int s = static_cast<int>(k % STAGES);
+        const uint32_t par = static_cast<uint32_t>((k / STAGES) & 1);
         unsigned char *st = stage0 + s * lay.bytes;
         const int ntok = static_cast<int>(min64(kTile, len - k * kTile));
         const bool ok = mbar_wait(&full[s], par);
@@ -339,17 +525,17 @@ __global__ void __launch_bounds__(kMaxThreads, 3)
             // Give up on this chunk: record it, let issued copies land, leave.
             if (tid == 0) {
                 atomicOr(&g_scan_status, PRECOG_DEV_TIMEOUT);
-                for (int64_t kk = k; kk < min64(k + kStages, ntiles); ++kk)
-                    mbar_wait(&full[kk % kStages], static_cast<uint32_t>((kk / kStages) & 1));
+                for (int64_t kk2 = k; kk2 < min64(k + STAGES, ntiles); ++kk2)
+                    mbar_wait(&full[kk2 % STAGES], static_cast<uint32_t>((kk2 / STAGES) & 1));
             }
             return;
         }
-        if (use_pow)
-            scan_tile<TIn, HAS_Y, true>(st, lay, DS, dl, ntok, h, kpow, kgen, yrow, p.y_dtype,
-                                        y_stride);
-        else
-            scan_tile<TIn, HAS_Y, false>(st, lay, DS, dl, ntok, h, kpow, kgen, yrow, p.y_dtype,
-                                         y_stride);
+        if constexpr (RESCALED) {
+            scan_tile_rescaled<TIn>(st, lay, DS, dl, ntok, h, Lw, kk, wmask);
+        } else {
+            scan_tile<TIn, HAS_Y, MODE == kPower>(st, lay, DS, dl, ntok, h, kpow, kgen, yrow,
+                                                 p.y_dtype, y_stride);
+        }
         if (HAS_Y) {
             yrow = (p.y_dtype == PRECOG_F32)
                        ? static_cast<void *>(static_cast<float *>(yrow) + kTile * y_stride)
@@ -357,10 +543,14 @@ __global__ void __launch_bounds__(kMaxThreads, 3)
         }
         fence_proxy_async_smem();
         __syncthreads();
-        if (tid == 0 && k + kStages < ntiles) issue(k + kStages);
+        if (tid == 0 && k + STAGES < ntiles) issue(k + STAGES);
     }
 
     // ---- state capture ----
+    if constexpr (RESCALED) {
+#pragma unroll
+        for (int j = 0; j < kCPT; ++j) renormalise(h[j], Lw[j]);
+    }
     if (p.states) {
 #pragma unroll
         for (int j = 0; j < kCPT; ++j) {
@@ -378,32 +568,42 @@ int pick_slice(int D, int sz) {
     return 0;
 }
 
-template <typename TIn, bool HAS_Y, bool HAS_H0>
+template <typename TIn, bool HAS_Y, bool HAS_H0, int MODE>
 cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
     const int sz = sizeof(TIn);
     const int DS = pick_slice(p.D, sz);
     if (DS == 0) return cudaErrorInvalidValue;
     const int slices = p.D / DS;
     const StageLayout lay = stage_layout(DS, sz, HAS_Y, !std::is_same<TIn, float>::value);
-    const size_t smem = kBarBytes + static_cast<size_t>(kStages) * lay.bytes;
+    const size_t smem = kBarBytes + static_cast<size_t>(Shape<MODE, HAS_Y>::kStagesUsed) * lay.bytes;
     const int64_t items = static_cast<int64_t>(p.n_layers) * p.n_chunks * slices;
     if (items == 0) return cudaSuccess;
     if (items > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-    auto kern = scan_kernel<TIn, HAS_Y, HAS_H0>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
+    auto kern = scan_kernel<TIn, HAS_Y, HAS_H0, MODE>;
+    static int smem_set = 0;
+    cudaError_t e = ensure_smem(reinterpret_cast<const void *>(kern), &smem_set, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     kern<<<static_cast<unsigned>(items), DS / kCPT, smem, stream>>>(p, DS, slices);
-    return cudaGetLastError();
+    e = cudaGetLastError();
+    if (e == cudaSuccess) count_launches(1);
+    return e;
+}
+
+template <typename TIn, int MODE>
+cudaError_t launch_mode(const ScanParams &p, cudaStream_t stream) {
+    const bool has_y = p.y != nullptr;
+    const bool has_h0 = p.bank != nullptr;
+    if (has_y)
+        return has_h0 ? launch_t<TIn, true, true, MODE>(p, stream)
+                      : launch_t<TIn, true, false, MODE>(p, stream);
+    return has_h0 ? launch_t<TIn, false, true, MODE>(p, stream)
+                  : launch_t<TIn, false, false, MODE>(p, stream);
 }
 
 template <typename TIn>
 cudaError_t launch_in(const ScanParams &p, cudaStream_t stream) {
-    const bool has_y = p.y != nullptr;
-    const bool has_h0 = p.bank != nullptr;
-    if (has_y)
-        return has_h0 ? launch_t<TIn, true, true>(p, stream) : launch_t<TIn, true, false>(p, stream);
-    return has_h0 ? launch_t<TIn, false, true>(p, stream) : launch_t<TIn, false, false>(p, stream);
+    return p.a_kind == PRECOG_A_POWER ? launch_mode<TIn, kPower>(p, stream)
+                                      : launch_mode<TIn, kGeneral>(p, stream);
 }
 
 }  // namespace

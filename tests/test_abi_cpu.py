@@ -68,6 +68,7 @@ def _encode(lib, s, offsets=FAKE, n_chunks=4, T_tot=64, states=FAKE, sdt=0, laye
 @pytest.mark.parametrize("change,expect", [
     ({"N": 8}, 2), ({"D": 0}, 1), ({"D": 12}, 2), ({"in_dtype": 2}, 2), ({"x": 0}, 1),
     ({"A": FAKE + 4}, 1), ({"n_layers": 0}, 1), ({"n_layers": 2, "layer_stride_xd": 10}, 1),
+    ({"a_kind": 2}, 1), ({"a_kind": -1}, 1),
 ])
 def test_encode_rejects_bad_inputs(lib, change, expect):
     import paper_2608_02560_gb300 as pg

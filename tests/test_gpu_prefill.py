@@ -19,13 +19,19 @@ def _t(a, dev, dtype=None):
     return torch.from_numpy(np.ascontiguousarray(a)).to(dev, dtype or torch.float32)
 
 
-def test_theorem1_via_abi_bit_identical(cuda_device):
+@pytest.mark.parametrize("power,ctx_readout", [(False, True), (True, True), (True, False)])
+def test_theorem1_via_abi(cuda_device, power, ctx_readout):
     """Encode [chunk; query] from the zero state with readout, versus encode(chunk) then
-    prefill(query) from the captured fp32 state: identical operation sequence on the GPU,
-    so states and every query y_t agree bit for bit (Theorem 1, Proposition)."""
+    prefill(query) from the captured fp32 state (Theorem 1 and the Proposition).
+
+    When both encodes run the same update form (the readout variant) the GPU performs
+    the identical operation sequence, so the state and every query y_t agree bit for
+    bit. Capturing the chunk without readout under a structured A uses the rescaled
+    accumulation, whose rounding differs: then the agreement is within 1e-5."""
     import torch
     pg = _pg()
     d = cuda_device
+    kind = pg.PRECOG_A_POWER if power else pg.PRECOG_A_GENERAL
     D, N = 256, 16
     Lc, Tq = 413, 64
     x, dt, A, B, C = synth.host_scan_inputs(Lc + Tq, D, N, seed=123)
@@ -33,20 +39,27 @@ def test_theorem1_via_abi_bit_identical(cuda_device):
     xb, dtb, Bb, Cb, Ad = tb(x), tb(dt), tb(B), tb(C), _t(A, d)
     full_state = torch.empty((1, 1, D, N), dtype=torch.float32, device=d)
     full_y = torch.empty((1, Lc + Tq, D), dtype=torch.float32, device=d)
-    pg.precog_encode_chunks(pg.scan_inputs(xb, dtb, Bb, Ad, Cb),
+    pg.precog_encode_chunks(pg.scan_inputs(xb, dtb, Bb, Ad, Cb, a_kind=kind),
                             _t(np.array([0, Lc + Tq]), d, torch.int64), Lc + Tq,
                             states_out=full_state, y_out=full_y)
     ctx_state = torch.empty((1, 1, D, N), dtype=torch.float32, device=d)
-    pg.precog_encode_chunks(pg.scan_inputs(xb[:Lc], dtb[:Lc], Bb[:Lc], Ad),
-                            _t(np.array([0, Lc]), d, torch.int64), Lc, states_out=ctx_state)
+    ctx_y = torch.empty((1, Lc, D), dtype=torch.float32, device=d) if ctx_readout else None
+    pg.precog_encode_chunks(pg.scan_inputs(xb[:Lc], dtb[:Lc], Bb[:Lc], Ad, Cb[:Lc], a_kind=kind),
+                            _t(np.array([0, Lc]), d, torch.int64), Lc, states_out=ctx_state,
+                            y_out=ctx_y)
     q_y = torch.empty((1, Tq, D), dtype=torch.float32, device=d)
     q_state = torch.empty((1, 1, D, N), dtype=torch.float32, device=d)
     pg.precog_prefill_from_state(pg.scan_inputs(xb[Lc:].contiguous(), dtb[Lc:].contiguous(),
-                                                Bb[Lc:].contiguous(), Ad, Cb[Lc:].contiguous()),
+                                                Bb[Lc:].contiguous(), Ad, Cb[Lc:].contiguous(),
+                                                a_kind=kind),
                                  1, Tq, ctx_state, idx=None, y_out=q_y, state_out=q_state)
     assert pg.precog_device_status()[0] == 0
-    assert torch.equal(full_state, q_state)
-    assert torch.equal(full_y[:, Lc:], q_y)
+    if ctx_readout:
+        assert torch.equal(full_state, q_state)
+        assert torch.equal(full_y[:, Lc:], q_y)
+    else:
+        assert rel_err(to_np(q_state), to_np(full_state)) < TOL_F32
+        assert rel_err(to_np(q_y), to_np(full_y[:, Lc:])) < TOL_F32
     # and both agree with the oracle's in-context scan
     ref_h, ref_y = oracle.rollout(to_np(xb), to_np(dtb), A, to_np(Bb), to_np(Cb), want_y=True)
     assert rel_err(to_np(q_state[0, 0]), ref_h) < 1e-5
@@ -62,7 +75,8 @@ def test_tiny_end_to_end(cuda_device):
     w = synth.tiny_workload(0)
     D, N = w.A.shape
     bank = torch.empty((8, 1, D, N), dtype=torch.float32, device=d)
-    pg.precog_encode_chunks(pg.scan_inputs(_t(w.x, d), _t(w.dt, d), _t(w.B, d), _t(w.A, d)),
+    pg.precog_encode_chunks(pg.scan_inputs(_t(w.x, d), _t(w.dt, d), _t(w.B, d), _t(w.A, d),
+                                           a_kind=pg.PRECOG_A_POWER),
                             _t(w.offsets, d, torch.int64), w.x.shape[0], states_out=bank)
     idx = torch.empty(1, dtype=torch.int64, device=d)
     pg.precog_retrieve(_t(w.index, d), _t(w.query, d), idx)
@@ -126,8 +140,8 @@ def test_query_workload_prefill(cuda_device, Q):
     x, dt, B, C, A = stack("x"), stack("dt"), stack("B"), stack("C"), stack("A")
     y = torch.empty((L, Q * Tq, D), dtype=torch.bfloat16, device=d)
     h = torch.empty((Q, L, D, N), dtype=torch.bfloat16, device=d)
-    pg.precog_prefill_from_state(pg.scan_inputs(x, dt, B, A, C), Q, Tq, bank, idx=idx,
-                                 y_out=y, state_out=h)
+    pg.precog_prefill_from_state(pg.scan_inputs(x, dt, B, A, C, a_kind=pg.PRECOG_A_POWER), Q, Tq,
+                                 bank, idx=idx, y_out=y, state_out=h)
     assert pg.precog_device_status()[0] == 0
     An = A[0].cpu().numpy()
     for q in sorted({0, Q - 1, Q // 3}):

@@ -25,9 +25,10 @@ def _t(a, dev, dtype=None):
     return torch.from_numpy(np.ascontiguousarray(a)).to(dev, dtype or torch.float32)
 
 
-def _encode(dev, x, dt, B, A, offsets, C=None, state_dtype=None, y_dtype=None):
+def _encode(dev, x, dt, B, A, offsets, C=None, state_dtype=None, y_dtype=None, power=False):
     import torch
     pg = _pg()
+    kind = pg.PRECOG_A_POWER if power else pg.PRECOG_A_GENERAL
     n_chunks = offsets.numel() - 1
     L = 1 if x.dim() == 2 else x.shape[0]
     D, N = A.shape[-2], A.shape[-1]
@@ -37,23 +38,27 @@ def _encode(dev, x, dt, B, A, offsets, C=None, state_dtype=None, y_dtype=None):
     if y_dtype is not None:
         T = x.shape[-2]
         y = torch.zeros((L, T, D), dtype=y_dtype, device=dev)
-    pg.precog_encode_chunks(pg.scan_inputs(x, dt, B, A, C), offsets, x.shape[-2], states_out=states,
-                            y_out=y)
+    pg.precog_encode_chunks(pg.scan_inputs(x, dt, B, A, C, a_kind=kind), offsets, x.shape[-2],
+                            states_out=states, y_out=y)
     st, bits = pg.precog_device_status()
     assert st == 0, f"device status {st} bits {bits:#x}"
     return states, y
 
 
-def test_tiny_workload_fp32(cuda_device):
-    """1 layer, D=64, N=16, fp32, 8 chunks x 256 tokens: states and every y_t."""
+@pytest.mark.parametrize("power", [False, True])
+def test_tiny_workload_fp32(cuda_device, power):
+    """1 layer, D=64, N=16, fp32, 8 chunks x 256 tokens: states and every y_t (direct
+    update), and states alone (rescaled accumulation when A is stated structured)."""
     import torch
     w = synth.tiny_workload(0)
     d = cuda_device
-    states, y = _encode(d, _t(w.x, d), _t(w.dt, d), _t(w.B, d), _t(w.A, d),
-                        _t(w.offsets, d, torch.int64), C=_t(w.C, d), y_dtype=torch.float32)
+    args = (d, _t(w.x, d), _t(w.dt, d), _t(w.B, d), _t(w.A, d), _t(w.offsets, d, torch.int64))
+    states, y = _encode(*args, C=_t(w.C, d), y_dtype=torch.float32, power=power)
+    capt, _ = _encode(*args, power=power)
     ref_s, ref_y = oracle.scan(w.x, w.dt, w.A, w.B, w.offsets, C=w.C, want_y=True)
     for c in range(ref_s.shape[0]):
         assert rel_err(to_np(states[c, 0]), ref_s[c]) < TOL_F32
+        assert rel_err(to_np(capt[c, 0]), ref_s[c]) < TOL_F32
         s, e = w.offsets[c], w.offsets[c + 1]
         assert rel_err(to_np(y[0, s:e]), ref_y[s:e]) < TOL_F32
 
@@ -94,13 +99,17 @@ def test_A_zero_cumulative_sum_bit_exact(cuda_device):
     C = (rng.integers(-4, 5, size=(T, N)) / 4.0).astype(np.float32)
     A = np.zeros((D, N), dtype=np.float32)
     off = np.array([0, 77, T], dtype=np.int64)
-    states, y = _encode(d, _t(x, d), _t(dt, d), _t(B, d), _t(A, d), _t(off, d, torch.int64),
-                        C=_t(C, d), y_dtype=torch.float32)
-    for c in range(2):
-        s, e = off[c], off[c + 1]
-        traj = np.cumsum((dt[s:e] * x[s:e]).astype(np.float64)[:, :, None] * B[s:e, None, :], axis=0)
-        np.testing.assert_array_equal(to_np(states[c, 0]), traj[-1])
-        np.testing.assert_array_equal(to_np(y[0, s:e]), np.einsum("tn,tdn->td", C[s:e], traj))
+    args = (d, _t(x, d), _t(dt, d), _t(B, d), _t(A, d), _t(off, d, torch.int64))
+    for power in (False, True):
+        states, y = _encode(*args, C=_t(C, d), y_dtype=torch.float32, power=power)
+        capt, _ = _encode(*args, power=power)
+        for c in range(2):
+            s, e = off[c], off[c + 1]
+            traj = np.cumsum((dt[s:e] * x[s:e]).astype(np.float64)[:, :, None] * B[s:e, None, :],
+                             axis=0)
+            np.testing.assert_array_equal(to_np(states[c, 0]), traj[-1])
+            np.testing.assert_array_equal(to_np(capt[c, 0]), traj[-1])
+            np.testing.assert_array_equal(to_np(y[0, s:e]), np.einsum("tn,tdn->td", C[s:e], traj))
 
 
 def test_multi_layer_call_and_layer_offset(cuda_device):
@@ -118,8 +127,8 @@ def test_multi_layer_call_and_layer_offset(cuda_device):
     B = _t(np.stack([i[3] for i in ins]), d)
     A = _t(np.stack([synth.structured_A(D, N) * (1 + 0.5 * l) for l in range(L)]), d)
     bank = torch.full((2, 5, D, N), 7.0, dtype=torch.float32, device=d)
-    pg.precog_encode_chunks(pg.scan_inputs(x, dt, B, A), _t(off, d, torch.int64), T,
-                            states_out=bank, layer0=2, L_total=5)
+    pg.precog_encode_chunks(pg.scan_inputs(x, dt, B, A, a_kind=pg.PRECOG_A_POWER),
+                            _t(off, d, torch.int64), T, states_out=bank, layer0=2, L_total=5)
     assert pg.precog_device_status()[0] == 0
     got = to_np(bank)
     assert np.all(got[:, :2] == 7.0)
@@ -140,8 +149,8 @@ def test_bf16_capture_and_readout(cuda_device):
     tb = lambda a: _t(a, d, torch.bfloat16)
     xb, dtb, Bb, Cb = tb(x), tb(dt), tb(B), tb(C)
     s16, y16 = _encode(d, xb, dtb, Bb, _t(A, d), _t(off, d, torch.int64), C=Cb,
-                       state_dtype=torch.bfloat16, y_dtype=torch.bfloat16)
-    s32, _ = _encode(d, xb, dtb, Bb, _t(A, d), _t(off, d, torch.int64))
+                       state_dtype=torch.bfloat16, y_dtype=torch.bfloat16, power=True)
+    s32, _ = _encode(d, xb, dtb, Bb, _t(A, d), _t(off, d, torch.int64), power=True)
     ref_s, ref_y = oracle.scan(to_np(xb), to_np(dtb), A, to_np(Bb), off, C=to_np(Cb), want_y=True)
     for c in range(3):
         assert rel_err(to_np(s32[c, 0]), ref_s[c]) < 1e-5
@@ -174,9 +183,57 @@ def test_deterministic(cuda_device):
     x, dt, A, B, _ = synth.host_scan_inputs(512, 256, 16, seed=9)
     off = _t(np.array([0, 256, 512], dtype=np.int64), d, torch.int64)
     args = [_t(v, d, torch.bfloat16) for v in (x, dt, B)]
-    a, _ = _encode(d, args[0], args[1], args[2], _t(A, d), off)
-    b, _ = _encode(d, args[0], args[1], args[2], _t(A, d), off)
-    assert torch.equal(a, b)
+    for power in (False, True):
+        a, _ = _encode(d, args[0], args[1], args[2], _t(A, d), off, power=power)
+        b, _ = _encode(d, args[0], args[1], args[2], _t(A, d), off, power=power)
+        assert torch.equal(a, b)
+
+
+def test_power_statement_is_verified(cuda_device):
+    """a_kind = PRECOG_A_POWER with an A that is not (n+1)*A[d,0]: nothing is written for
+    the affected channel blocks and PRECOG_DEV_BAD_A is flagged; A[d,0] > 0 as well."""
+    import torch
+    pg = _pg()
+    d = cuda_device
+    T, D, N = 50, 512, 16
+    x, dt, A, B, _ = synth.host_scan_inputs(T, D, N, seed=2)
+    A_bad = A.copy()
+    A_bad[300, 5] *= 1.5                    # channel 300 sits in the second 256-channel block
+    off = _t(np.array([0, T], dtype=np.int64), d, torch.int64)
+    for Ab in (A_bad, -A):
+        states = torch.full((1, 1, D, N), 3.0, dtype=torch.float32, device=d)
+        pg.precog_encode_chunks(pg.scan_inputs(_t(x, d), _t(dt, d), _t(B, d), _t(Ab, d),
+                                               a_kind=pg.PRECOG_A_POWER), off, T, states_out=states)
+        st, bits = pg.precog_device_status()
+        assert st == 5 and bits == pg.PRECOG_DEV_BAD_A
+        assert torch.all(states[0, 0, 256:] == 3.0)
+    ref, _ = oracle.rollout(x, dt, A, B)
+    states = torch.full((1, 1, D, N), 3.0, dtype=torch.float32, device=d)
+    pg.precog_encode_chunks(pg.scan_inputs(_t(x, d), _t(dt, d), _t(B, d), _t(A_bad, d),
+                                           a_kind=pg.PRECOG_A_POWER), off, T, states_out=states)
+    pg.precog_device_status()
+    assert rel_err(to_np(states[0, 0, :256]), ref[:256]) < TOL_F32   # the valid block is done
+
+
+@pytest.mark.parametrize("scale,dt_shift", [(1.0, -2.0), (40.0, -2.0), (1.0, 2.5), (0.02, -4.0)])
+def test_rescaled_renormalisation_regimes(cuda_device, scale, dt_shift):
+    """The rescaled accumulation against the oracle where renormalisation is frequent
+    (large |A| or large dt: single tokens that decay past the window go through the
+    direct update), rare (tiny |A|, long memory) or mixed, fp32 inputs, 1e-5."""
+    import torch
+    d = cuda_device
+    T, D, N = 1500, 64, 16
+    rng = np.random.default_rng(int(scale * 100) + 7)
+    x = rng.standard_normal((T, D)).astype(np.float32)
+    dt = np.logaddexp(0.0, rng.standard_normal((T, D)) + dt_shift).astype(np.float32)
+    B = (rng.standard_normal((T, N)) * 0.25).astype(np.float32)
+    A = (synth.structured_A(D, N) * scale).astype(np.float32)
+    off = np.array([0, 700, 701, T], dtype=np.int64)
+    capt, _ = _encode(d, _t(x, d), _t(dt, d), _t(B, d), _t(A, d), _t(off, d, torch.int64),
+                      power=True)
+    ref, _ = oracle.scan(x, dt, A, B, off)
+    for c in range(3):
+        assert rel_err(to_np(capt[c, 0]), ref[c]) < TOL_F32, c
 
 
 # ------------------------------------------------------------- full-size workloads, sampled
@@ -195,7 +252,8 @@ def _sampled_check(dev, shape, layer, sample_chunks, y_mode=False, seed=0):
                          device=dev)
     y = torch.empty((1, T, shape.D), dtype=torch.bfloat16, device=dev) if y_mode else None
     pg.precog_encode_chunks(pg.scan_inputs(inp["x"], inp["dt"], inp["B"], inp["A"],
-                                           inp.get("C") if y_mode else None),
+                                           inp.get("C") if y_mode else None,
+                                           a_kind=pg.PRECOG_A_POWER),
                             off, T, states_out=states, layer0=layer, L_total=shape.n_layers,
                             y_out=y)
     assert pg.precog_device_status()[0] == 0
