@@ -206,8 +206,10 @@ def run_case(args):
     res = {"case": args.case}
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
     if args.case == "scan-small":
-        shape, chunks = synth.PAPER, 512
-        off_np = synth.fixed_offsets(chunks, shape.chunk_len)
+        # paper-shaped rows (D=256, N=16, bf16) in 3040 chunks of 1000 tokens: 3.2 GB, about
+        # 20 blocks per SM, so the per-token behaviour and occupancy match the full launch
+        shape, chunks, clen = synth.PAPER, 3040, 1000
+        off_np = synth.fixed_offsets(chunks, clen)
         T = int(off_np[-1])
         inp = synth.device_scan_inputs(T, shape.D, shape.N, 0, 0, dev, with_C=False)
         bank = torch.empty((chunks, shape.n_layers, shape.D, shape.N), dtype=torch.bfloat16, device=dev)
@@ -215,7 +217,7 @@ def run_case(args):
         si = pg.scan_inputs(inp["x"], inp["dt"], inp["B"], inp["A"], a_kind=pg.PRECOG_A_POWER)
         fn = lambda: pg.precog_encode_chunks(si, off, T, states_out=bank, layer0=0, L_total=shape.n_layers)
         res["algorithmic_bytes_per_launch"] = scan_bytes_per_launch(T, chunks, shape.D, shape.N)
-        res["scale_to_full_launch"] = shape.n_chunks / chunks
+        res["scale_to_full_launch"] = shape.n_chunks * shape.chunk_len / T
     elif args.case == "retrieve-small":
         M = 1 << 18
         index = synth.device_unit_index(M, synth.QUERY_DIM, 0, dev)

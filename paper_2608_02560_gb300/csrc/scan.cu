@@ -2,18 +2,21 @@
 // injected initial state (query prefill) -- Sec. 3 Eq. 1, Sec. 4.2, Eq. 2.
 //
 // Work decomposition: one CTA per (layer, chunk, slice of DS channels). Each
-// thread owns kCPT adjacent channels and keeps their N = 16 fp32 states in
+// thread owns CPT adjacent channels and keeps their N = 16 fp32 states in
 // registers for the whole chunk. The chunk's rows of x and dt (DS channels
-// each) and of B (and C) are staged into shared memory kTile tokens at a
-// time by the TMA engine (1-D bulk copies completing on an mbarrier), in a
-// kStages-deep ring, so the time loop only reads shared memory.
+// each) and of B (and C) are staged into shared memory TILE tokens at a time
+// by the TMA engine (1-D bulk copies completing on an mbarrier), in a
+// STAGES-deep ring, so the time loop only reads shared memory.
 //
-// Per token and channel the update is, for the 16 state indices n,
-//   h[n] <- alpha_n * h[n] + (dt * x) * B[n],   alpha_n = exp(dt * A[d, n]),
-// done as 8 packed fp32x2 multiply + 8 packed fp32x2 FMAs. When A[d, n] is
-// (n + 1) * A[d, 0] for every n (checked per CTA), alpha_n = r^(n+1) with
-// r = exp(dt * A[d, 0]): one SFU exponential per channel and a packed power
-// chain instead of 16 exponentials.
+// Per token and channel the recurrence is, for the 16 state indices n,
+//   h[n] <- alpha_n * h[n] + (dt * x) * B[n],   alpha_n = exp(dt * A[d, n]).
+// Three update forms, all in packed fp32x2 arithmetic:
+//   kGeneral   one SFU exponential per (d, n);
+//   kPower     A[d, n] = (n + 1) * A[d, 0] (stated by the caller, verified per
+//              CTA): alpha_n = r^(n+1), r = exp(dt * A[d, 0]), one exponential
+//              and a power chain per (t, d); with a readout y the state is
+//              updated directly, without one it is accumulated rescaled
+//              (see scan_tile_rescaled), which drops the per-n decay multiply.
 #include <type_traits>
 
 #include "../../include/precog.h"
@@ -25,49 +28,106 @@ namespace {
 
 __device__ uint32_t g_scan_status;
 
+// Shape of the rescaled capture kernel (channels per thread, tokens per stage,
+// stages, resident blocks per SM for the register budget).
+#ifndef PRECOG_RESCALED_CPT
+#define PRECOG_RESCALED_CPT 4
+#define PRECOG_RESCALED_TILE 16
+#define PRECOG_RESCALED_STAGES 2
+#define PRECOG_RESCALED_MINB 6
+#endif
+
 constexpr int kN = 16;          // state size (N) supported by the kernels
-constexpr int kCPT = 2;         // channels per thread
-constexpr int kTile = 16;       // tokens per pipeline stage
-constexpr int kStages = 4;      // pipeline depth
-constexpr int kMaxThreads = 128;
+constexpr int kMaxSlice = 256;  // channels per CTA at most
 constexpr int kBarBytes = 128;  // barrier area at the start of shared memory
 constexpr float kLog2e = 1.4426950408889634f;
 
 __device__ __forceinline__ int64_t min64(int64_t a, int64_t b) { return a < b ? a : b; }
 
+enum Mode { kGeneral = 0, kPower = 1 };
+
+// Compile-time shape of one kernel instantiation.
+template <typename TIn_, bool HAS_Y_, bool HAS_H0_, int MODE_, int CPT_, int TILE_, int STAGES_,
+          int MINB_>
+struct Cfg {
+    using TIn = TIn_;
+    static constexpr bool HAS_Y = HAS_Y_, HAS_H0 = HAS_H0_;
+    static constexpr int MODE = MODE_, CPT = CPT_, TILE = TILE_, STAGES = STAGES_, MINB = MINB_;
+    static constexpr bool CONV = !std::is_same<TIn_, float>::value;
+    static constexpr int SZ = sizeof(TIn_);
+    static constexpr bool RESCALED = MODE_ == kPower && !HAS_Y_;
+};
+
 struct StageLayout {
     uint32_t xs, dts, bs, cs, bf, cf, bytes;
 };
 
-__host__ __device__ inline StageLayout stage_layout(int DS, int sz, bool has_y, bool conv) {
+__host__ __device__ inline StageLayout stage_layout(int tile, int DS, int sz, bool has_y, bool conv) {
     StageLayout L;
     uint32_t o = 0;
     L.xs = o;
-    o += kTile * DS * sz;
+    o += tile * DS * sz;
     L.dts = o;
-    o += kTile * DS * sz;
+    o += tile * DS * sz;
     L.bs = o;
-    o += kTile * kN * sz;
+    o += tile * kN * sz;
     L.cs = o;
-    if (has_y) o += kTile * kN * sz;
+    if (has_y) o += tile * kN * sz;
     L.bf = o;
-    if (conv) o += kTile * kN * 4;
+    if (conv) o += tile * kN * 4;
     L.cf = o;
-    if (conv && has_y) o += kTile * kN * 4;
+    if (conv && has_y) o += tile * kN * 4;
     L.bytes = (o + 127u) & ~127u;
     return L;
 }
 
-template <typename TIn>
-__device__ __forceinline__ void load_pair(const unsigned char *p, float &a, float &b) {
+// CPT adjacent channel values of one token row in shared memory; `neg` gets
+// the sign bits of the raw values (nonzero if any is negative).
+template <typename TIn, int CPT>
+__device__ __forceinline__ void load_chan(const unsigned char *p, float (&v)[CPT], uint32_t &neg) {
     if constexpr (std::is_same<TIn, float>::value) {
-        const float2 v = *reinterpret_cast<const float2 *>(p);
-        a = v.x;
-        b = v.y;
+        if constexpr (CPT == 2) {
+            const float2 q = *reinterpret_cast<const float2 *>(p);
+            v[0] = q.x;
+            v[1] = q.y;
+        } else {
+            const float4 q = *reinterpret_cast<const float4 *>(p);
+            v[0] = q.x;
+            v[1] = q.y;
+            v[2] = q.z;
+            v[3] = q.w;
+        }
+        uint32_t s = 0;
+#pragma unroll
+        for (int j = 0; j < CPT; ++j) s |= __float_as_uint(v[j]);
+        neg = s & 0x80000000u;
     } else {
-        const __nv_bfloat162 v = *reinterpret_cast<const __nv_bfloat162 *>(p);
-        a = __low2float(v);
-        b = __high2float(v);
+        uint32_t w[CPT / 2];
+        if constexpr (CPT == 2) {
+            w[0] = *reinterpret_cast<const uint32_t *>(p);
+        } else {
+            const uint2 q = *reinterpret_cast<const uint2 *>(p);
+            w[0] = q.x;
+            w[1] = q.y;
+        }
+        uint32_t s = 0;
+#pragma unroll
+        for (int i = 0; i < CPT / 2; ++i) {
+            v[2 * i] = __uint_as_float(w[i] << 16);
+            v[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+            s |= w[i];
+        }
+        neg = s & 0x80008000u;
+    }
+}
+
+__device__ __forceinline__ void load_b(const float *bsrc, int t, f2 (&b)[8]) {
+    const ulonglong2 *bv = reinterpret_cast<const ulonglong2 *>(bsrc + t * kN);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const ulonglong2 v = bv[i];
+        b[2 * i] = v.x;
+        b[2 * i + 1] = v.y;
     }
 }
 
@@ -127,43 +187,42 @@ __device__ __forceinline__ void load_state16(const void *base, int dtype, int64_
     for (int i = 0; i < 8; ++i) h[i] = pack2(v[2 * i], v[2 * i + 1]);
 }
 
-// Roll kTile (or fewer) tokens of one stage through the recurrence.
-template <typename TIn, bool HAS_Y, bool POW>
-__device__ __forceinline__ void scan_tile(const unsigned char *st, const StageLayout &lay, int DS,
-                                          int dl, int ntok, f2 (&h)[kCPT][8],
-                                          const float (&kpow)[kCPT], const f2 (&kgen)[kCPT][8],
-                                          void *yrow, int y_dtype, int64_t y_stride) {
-    constexpr bool CONV = !std::is_same<TIn, float>::value;
-    constexpr int sz = sizeof(TIn);
-    const float *bsrc = reinterpret_cast<const float *>(st + (CONV ? lay.bf : lay.bs));
-    const float *csrc = reinterpret_cast<const float *>(st + (CONV ? lay.cf : lay.cs));
+// p[i] = (r^(2i+1), r^(2i+2)) for i = 0..7
+__device__ __forceinline__ void pow_pairs(float r, f2 (&p)[8]) {
+    const float r2 = r * r;
+    p[0] = pack2(r, r2);
+    const f2 rr = pack2(r2, r2);
+#pragma unroll
+    for (int i = 1; i < 8; ++i) p[i] = mul2(p[i - 1], rr);
+}
+
+// ---------------------------------------------------------------------------
+// Direct update (any readout): h_n <- alpha_n h_n + u B_n, y = sum_n C_n h_n.
+template <class C>
+__device__ __forceinline__ void scan_tile_direct(const unsigned char *st, const StageLayout &lay,
+                                                 int DS, int dl, int ntok,
+                                                 f2 (&h)[C::CPT][8], const float (&kpow)[C::CPT],
+                                                 const f2 (&kgen)[C::CPT][8], void *yrow,
+                                                 int y_dtype, int64_t y_stride) {
+    constexpr int CPT = C::CPT;
+    const float *bsrc = reinterpret_cast<const float *>(st + (C::CONV ? lay.bf : lay.bs));
+    const float *csrc = reinterpret_cast<const float *>(st + (C::CONV ? lay.cf : lay.cs));
     for (int t = 0; t < ntok; ++t) {
         f2 b[8];
-        const ulonglong2 *bv = reinterpret_cast<const ulonglong2 *>(bsrc + t * kN);
+        load_b(bsrc, t, b);
+        float xv[CPT], dv[CPT], yv[CPT];
+        uint32_t neg;
+        load_chan<typename C::TIn, CPT>(st + lay.xs + (t * DS + dl) * C::SZ, xv, neg);
+        load_chan<typename C::TIn, CPT>(st + lay.dts + (t * DS + dl) * C::SZ, dv, neg);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const ulonglong2 v = bv[i];
-            b[2 * i] = v.x;
-            b[2 * i + 1] = v.y;
-        }
-        float xv[kCPT], dv[kCPT];
-        load_pair<TIn>(st + lay.xs + (t * DS + dl) * sz, xv[0], xv[1]);
-        load_pair<TIn>(st + lay.dts + (t * DS + dl) * sz, dv[0], dv[1]);
-        float yv[kCPT];
-#pragma unroll
-        for (int j = 0; j < kCPT; ++j) {
+        for (int j = 0; j < CPT; ++j) {
             const float u = dv[j] * xv[j];
             const f2 uu = pack2(u, u);
-            if constexpr (POW) {
-                const float r = ex2(dv[j] * kpow[j]);
-                const float r2 = r * r;
-                f2 aa = pack2(r, r2);
-                const f2 rr = pack2(r2, r2);
+            if constexpr (C::MODE == kPower) {
+                f2 a[8];
+                pow_pairs(ex2(dv[j] * kpow[j]), a);
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    if (i) aa = mul2(aa, rr);
-                    h[j][i] = fma2(aa, h[j][i], mul2(uu, b[i]));
-                }
+                for (int i = 0; i < 8; ++i) h[j][i] = fma2(a[i], h[j][i], mul2(uu, b[i]));
             } else {
                 const f2 dd = pack2(dv[j], dv[j]);
 #pragma unroll
@@ -173,7 +232,7 @@ __device__ __forceinline__ void scan_tile(const unsigned char *st, const StageLa
                     h[j][i] = fma2(pack2(ex2(e0), ex2(e1)), h[j][i], mul2(uu, b[i]));
                 }
             }
-            if constexpr (HAS_Y) {
+            if constexpr (C::HAS_Y) {
                 const ulonglong2 *cv = reinterpret_cast<const ulonglong2 *>(csrc + t * kN);
                 f2 acc = 0;
 #pragma unroll
@@ -187,14 +246,24 @@ __device__ __forceinline__ void scan_tile(const unsigned char *st, const StageLa
                 yv[j] = lo + hi;
             }
         }
-        if constexpr (HAS_Y) {
+        if constexpr (C::HAS_Y) {
             if (y_dtype == PRECOG_F32) {
-                float2 *dst = reinterpret_cast<float2 *>(static_cast<float *>(yrow) + t * y_stride);
-                *dst = make_float2(yv[0], yv[1]);
+                float *dst = static_cast<float *>(yrow) + t * y_stride;
+                if constexpr (CPT == 2) {
+                    *reinterpret_cast<float2 *>(dst) = make_float2(yv[0], yv[1]);
+                } else {
+                    *reinterpret_cast<float4 *>(dst) = make_float4(yv[0], yv[1], yv[2], yv[3]);
+                }
             } else {
-                __nv_bfloat162 *dst = reinterpret_cast<__nv_bfloat162 *>(
-                    static_cast<__nv_bfloat16 *>(yrow) + t * y_stride);
-                *dst = __floats2bfloat162_rn(yv[0], yv[1]);
+                __nv_bfloat16 *dst = static_cast<__nv_bfloat16 *>(yrow) + t * y_stride;
+                __nv_bfloat162 p0 = __floats2bfloat162_rn(yv[0], yv[1]);
+                if constexpr (CPT == 2) {
+                    *reinterpret_cast<__nv_bfloat162 *>(dst) = p0;
+                } else {
+                    __nv_bfloat162 p1 = __floats2bfloat162_rn(yv[2], yv[3]);
+                    *reinterpret_cast<uint2 *>(dst) = make_uint2(
+                        *reinterpret_cast<uint32_t *>(&p0), *reinterpret_cast<uint32_t *>(&p1));
+                }
             }
         }
     }
@@ -207,19 +276,11 @@ __device__ __forceinline__ void scan_tile(const unsigned char *st, const StageLa
 //   G_n += (u * E_t^(n+1)) * B_n,     u = dt * x,
 // so the per-n decay multiply of the direct update disappears: per token and
 // channel one exponential, a packed power chain and 16 FMAs. Whenever some
-// lane's L would pass kLmax the whole warp renormalises (h_n = G_n E^-(n+1),
-// L = 0), which keeps E^16 <= 2^(16 * kLmax) far from fp32 overflow. A single
-// token whose own increment exceeds kLmax is applied directly to h.
+// lane's L would leave [-kLmax, kLmax] the whole warp renormalises
+// (h_n = G_n E^-(n+1), L = 0), which keeps E^(+-16) within 2^(16 * kLmax),
+// far from fp32 overflow and underflow. A single token whose own increment is
+// outside the window is applied to h directly.
 constexpr float kLmax = 6.0f;
-
-// p[i] = (r^(2i+1), r^(2i+2)) for i = 0..7
-__device__ __forceinline__ void pow_pairs(float r, f2 (&p)[8]) {
-    const float r2 = r * r;
-    p[0] = pack2(r, r2);
-    const f2 rr = pack2(r2, r2);
-#pragma unroll
-    for (int i = 1; i < 8; ++i) p[i] = mul2(p[i - 1], rr);
-}
 
 __device__ __forceinline__ void renormalise(f2 (&g)[8], float &L) {
     f2 p[8];
@@ -244,24 +305,23 @@ __device__ __forceinline__ void accumulate(f2 (&g)[8], const f2 (&b)[8], float u
     }
 }
 
-// One token with the window check: renormalise the whole warp when some lane
-// would leave [-kLmax, kLmax]; a token whose own increment is outside it is
-// applied to h directly (alpha_n = 2^(-(n+1)*Ln)) and contributes nothing to G.
-__device__ __forceinline__ void token_checked(f2 (&g)[kCPT][8], float (&L)[kCPT],
-                                              const float (&kk)[kCPT], const f2 (&b)[8],
-                                              const float (&xv)[kCPT], const float (&dv)[kCPT],
+// One token with the window check of every lane and channel.
+template <int CPT>
+__device__ __forceinline__ void token_checked(f2 (&g)[CPT][8], float (&L)[CPT],
+                                              const float (&kk)[CPT], const f2 (&b)[8],
+                                              const float (&xv)[CPT], const float (&dv)[CPT],
                                               unsigned wmask) {
-    float Ln[kCPT], u[kCPT];
+    float Ln[CPT], u[CPT];
     bool need = false;
 #pragma unroll
-    for (int j = 0; j < kCPT; ++j) {
+    for (int j = 0; j < CPT; ++j) {
         Ln[j] = fmaf(dv[j], kk[j], L[j]);
         u[j] = dv[j] * xv[j];
         need |= !(fabsf(Ln[j]) <= kLmax);
     }
     if (__any_sync(wmask, need)) {
 #pragma unroll
-        for (int j = 0; j < kCPT; ++j) {
+        for (int j = 0; j < CPT; ++j) {
             renormalise(g[j], L[j]);
             Ln[j] = dv[j] * kk[j];
             if (!(fabsf(Ln[j]) <= kLmax)) {
@@ -276,109 +336,90 @@ __device__ __forceinline__ void token_checked(f2 (&g)[kCPT][8], float (&L)[kCPT]
         }
     }
 #pragma unroll
-    for (int j = 0; j < kCPT; ++j) {
+    for (int j = 0; j < CPT; ++j) {
         accumulate(g[j], b, u[j], Ln[j]);
         L[j] = Ln[j];
     }
 }
 
-template <typename TIn>
-__device__ __forceinline__ void load_token(const unsigned char *st, const StageLayout &lay,
-                                           const float *bsrc, int DS, int dl, int t, f2 (&b)[8],
-                                           float (&xv)[kCPT], float (&dv)[kCPT]) {
-    constexpr int sz = sizeof(TIn);
-    const ulonglong2 *bv = reinterpret_cast<const ulonglong2 *>(bsrc + t * kN);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const ulonglong2 v = bv[i];
-        b[2 * i] = v.x;
-        b[2 * i + 1] = v.y;
-    }
-    load_pair<TIn>(st + lay.xs + (t * DS + dl) * sz, xv[0], xv[1]);
-    load_pair<TIn>(st + lay.dts + (t * DS + dl) * sz, dv[0], dv[1]);
-}
-
-// Tokens go in groups of kGroup: the exponents of the whole group are summed
-// first (one serial FMA per token), one warp vote decides whether the group
-// stays inside the window, and then the group's accumulations carry no branch,
-// so the scheduler can interleave the power chains of its tokens.
+// Tokens go in groups of kGroup. The group's exponents are summed first (one
+// serial FMA per token and channel). With dt >= 0 they only grow, so checking
+// the group's last exponent covers every token in it; a negative dt anywhere
+// in the group (seen from the sign bits) sends the group through the per-token
+// check. One warp vote per group; the fast path then carries no branch, so the
+// power chains of the group's tokens can interleave.
 constexpr int kGroup = 4;
 
-template <typename TIn>
+template <class C>
 __device__ __forceinline__ void scan_tile_rescaled(const unsigned char *st, const StageLayout &lay,
-                                                   int DS, int dl, int ntok, f2 (&g)[kCPT][8],
-                                                   float (&L)[kCPT], const float (&kk)[kCPT],
-                                                   unsigned wmask) {
-    constexpr bool CONV = !std::is_same<TIn, float>::value;
-    constexpr int sz = sizeof(TIn);
-    const float *bsrc = reinterpret_cast<const float *>(st + (CONV ? lay.bf : lay.bs));
+                                                   int DS, int dl, int ntok,
+                                                   f2 (&g)[C::CPT][8], float (&L)[C::CPT],
+                                                   const float (&kk)[C::CPT], unsigned wmask) {
+    constexpr int CPT = C::CPT;
+    using TIn = typename C::TIn;
+    const float *bsrc = reinterpret_cast<const float *>(st + (C::CONV ? lay.bf : lay.bs));
     int t = 0;
     for (; t + kGroup <= ntok; t += kGroup) {
-        float Lk[kGroup][kCPT];
-        bool need = false;
+        float dvk[kGroup][CPT], Lk[kGroup][CPT];
+        uint32_t neg = 0;
 #pragma unroll
         for (int k = 0; k < kGroup; ++k) {
-            float dv[kCPT], xv[kCPT];
-            load_pair<TIn>(st + lay.dts + ((t + k) * DS + dl) * sz, dv[0], dv[1]);
+            uint32_t nk;
+            load_chan<TIn, CPT>(st + lay.dts + ((t + k) * DS + dl) * C::SZ, dvk[k], nk);
+            neg |= nk;
 #pragma unroll
-            for (int j = 0; j < kCPT; ++j) {
-                Lk[k][j] = fmaf(dv[j], kk[j], k ? Lk[k - 1][j] : L[j]);
-                need |= !(fabsf(Lk[k][j]) <= kLmax);
-            }
-            (void)xv;
+            for (int j = 0; j < CPT; ++j) Lk[k][j] = fmaf(dvk[k][j], kk[j], k ? Lk[k - 1][j] : L[j]);
         }
+        bool need = neg != 0;
+#pragma unroll
+        for (int j = 0; j < CPT; ++j) need |= !(fabsf(Lk[kGroup - 1][j]) <= kLmax);
         if (__any_sync(wmask, need)) {
-#pragma unroll 1
+            // unrolled so that dvk stays in registers (no dynamic indexing)
+#pragma unroll
             for (int k = 0; k < kGroup; ++k) {
                 f2 b[8];
-                float xv[kCPT], dv[kCPT];
-                load_token<TIn>(st, lay, bsrc, DS, dl, t + k, b, xv, dv);
-                token_checked(g, L, kk, b, xv, dv, wmask);
+                float xv[CPT];
+                uint32_t nx;
+                load_b(bsrc, t + k, b);
+                load_chan<TIn, CPT>(st + lay.xs + ((t + k) * DS + dl) * C::SZ, xv, nx);
+                token_checked<CPT>(g, L, kk, b, xv, dvk[k], wmask);
             }
         } else {
 #pragma unroll
             for (int k = 0; k < kGroup; ++k) {
                 f2 b[8];
-                float xv[kCPT], dv[kCPT];
-                load_token<TIn>(st, lay, bsrc, DS, dl, t + k, b, xv, dv);
+                float xv[CPT];
+                uint32_t nx;
+                load_b(bsrc, t + k, b);
+                load_chan<TIn, CPT>(st + lay.xs + ((t + k) * DS + dl) * C::SZ, xv, nx);
 #pragma unroll
-                for (int j = 0; j < kCPT; ++j) accumulate(g[j], b, dv[j] * xv[j], Lk[k][j]);
+                for (int j = 0; j < CPT; ++j) accumulate(g[j], b, dvk[k][j] * xv[j], Lk[k][j]);
             }
 #pragma unroll
-            for (int j = 0; j < kCPT; ++j) L[j] = Lk[kGroup - 1][j];
+            for (int j = 0; j < CPT; ++j) L[j] = Lk[kGroup - 1][j];
         }
     }
     for (; t < ntok; ++t) {
         f2 b[8];
-        float xv[kCPT], dv[kCPT];
-        load_token<TIn>(st, lay, bsrc, DS, dl, t, b, xv, dv);
-        token_checked(g, L, kk, b, xv, dv, wmask);
+        float xv[CPT], dv[CPT];
+        uint32_t n0;
+        load_b(bsrc, t, b);
+        load_chan<TIn, CPT>(st + lay.xs + (t * DS + dl) * C::SZ, xv, n0);
+        load_chan<TIn, CPT>(st + lay.dts + (t * DS + dl) * C::SZ, dv, n0);
+        token_checked<CPT>(g, L, kk, b, xv, dv, wmask);
     }
 }
 
-// Update form of one kernel instantiation. kGeneral: one exponential per
-// (d, n). kPower: A[d, n] = (n + 1) * A[d, 0] (the caller states it, every CTA
-// verifies it): with readout, the direct update with a packed power chain;
-// without readout, the rescaled accumulation above.
-enum Mode { kGeneral = 0, kPower = 1 };
-
-template <int MODE, bool HAS_Y> struct Shape {
-    static constexpr bool kRescaled = MODE == kPower && !HAS_Y;
-    static constexpr int kStagesUsed = kRescaled ? 2 : kStages;
-    static constexpr int kMinBlocks = kRescaled ? 4 : 3;
-};
-
-template <typename TIn, bool HAS_Y, bool HAS_H0, int MODE>
-__global__ void __launch_bounds__(kMaxThreads, (Shape<MODE, HAS_Y>::kMinBlocks))
+// ---------------------------------------------------------------------------
+template <class C>
+__global__ void __launch_bounds__(kMaxSlice / C::CPT, C::MINB)
     scan_kernel(const ScanParams p, const int DS, const int slices) {
+    using TIn = typename C::TIn;
+    constexpr int CPT = C::CPT, TILE = C::TILE, STAGES = C::STAGES, SZ = C::SZ;
     extern __shared__ __align__(128) unsigned char smem[];
-    constexpr int sz = sizeof(TIn);
-    constexpr bool CONV = !std::is_same<TIn, float>::value;
-    constexpr bool RESCALED = Shape<MODE, HAS_Y>::kRescaled;
-    constexpr int STAGES = Shape<MODE, HAS_Y>::kStagesUsed;
     uint64_t *full = reinterpret_cast<uint64_t *>(smem);
     unsigned char *stage0 = smem + kBarBytes;
-    const StageLayout lay = stage_layout(DS, sz, HAS_Y, CONV);
+    const StageLayout lay = stage_layout(TILE, DS, SZ, C::HAS_Y, C::CONV);
     const int tid = threadIdx.x;
     const int nthr = blockDim.x;
 
@@ -402,30 +443,30 @@ __global__ void __launch_bounds__(kMaxThreads, (Shape<MODE, HAS_Y>::kMinBlocks))
         len = end - start;
     }
     const int d0 = slice * DS;
-    const int dl = tid * kCPT;
+    const int dl = tid * CPT;
     const int D = p.D;
     const TIn *xl = static_cast<const TIn *>(p.x) + layer * p.ls_xd;
     const TIn *dtl = static_cast<const TIn *>(p.dt) + layer * p.ls_xd;
     const TIn *Bl = static_cast<const TIn *>(p.B) + layer * p.ls_bc;
-    const TIn *Cl = HAS_Y ? static_cast<const TIn *>(p.C) + layer * p.ls_bc : nullptr;
+    const TIn *Cl = C::HAS_Y ? static_cast<const TIn *>(p.C) + layer * p.ls_bc : nullptr;
     const float *Al = p.A + static_cast<int64_t>(layer) * D * kN;
 
     // ---- coefficients; kPower verifies the structure before any copy is issued ----
-    float kpow[kCPT];                      // A[d, 0] * log2 e
-    f2 kgen[kCPT][8];                      // (A[d, n] * log2 e) pairs, kGeneral only
+    float kpow[CPT];      // A[d, 0] * log2 e
+    f2 kgen[CPT][8];      // (A[d, n] * log2 e) pairs, kGeneral only
 #pragma unroll
-    for (int j = 0; j < kCPT; ++j) {
+    for (int j = 0; j < CPT; ++j) {
         const float *a = Al + static_cast<int64_t>(d0 + dl + j) * kN;
         kpow[j] = a[0] * kLog2e;
-        if constexpr (MODE == kGeneral) {
+        if constexpr (C::MODE == kGeneral) {
 #pragma unroll
             for (int i = 0; i < 8; ++i) kgen[j][i] = pack2(a[2 * i] * kLog2e, a[2 * i + 1] * kLog2e);
         }
     }
-    if constexpr (MODE == kPower) {
+    if constexpr (C::MODE == kPower) {
         bool ok = true;
 #pragma unroll
-        for (int j = 0; j < kCPT; ++j) {
+        for (int j = 0; j < CPT; ++j) {
             const float *a = Al + static_cast<int64_t>(d0 + dl + j) * kN;
             const float a0 = a[0];
             ok &= a0 <= 0.f;
@@ -439,7 +480,7 @@ __global__ void __launch_bounds__(kMaxThreads, (Shape<MODE, HAS_Y>::kMinBlocks))
     }
 
     // ---- pipeline start: barrier init, first STAGES tiles in flight ----
-    const int64_t ntiles = (len + kTile - 1) / kTile;
+    const int64_t ntiles = (len + TILE - 1) / TILE;
     if (tid == 0) {
         for (int s = 0; s < STAGES; ++s) mbar_init(&full[s], 1);
         fence_barrier_init();
@@ -448,10 +489,10 @@ __global__ void __launch_bounds__(kMaxThreads, (Shape<MODE, HAS_Y>::kMinBlocks))
     auto issue = [&](int64_t k) {  // thread 0 only
         const int s = static_cast<int>(k % STAGES);
         unsigned char *st = stage0 + s * lay.bytes;
-        const int64_t row0 = start + k * kTile;
-        const int ntok = static_cast<int>(min64(kTile, len - k * kTile));
-        const uint32_t rowb = DS * sz;
-        const uint32_t bytes = ntok * rowb * 2 + ntok * kN * sz * (HAS_Y ? 2 : 1);
+        const int64_t row0 = start + k * TILE;
+        const int ntok = static_cast<int>(min64(TILE, len - k * TILE));
+        const uint32_t rowb = DS * SZ;
+        const uint32_t bytes = ntok * rowb * 2 + ntok * kN * SZ * (C::HAS_Y ? 2 : 1);
         mbar_arrive_expect_tx(&full[s], bytes);
         if (DS == D) {
             bulk_g2s(st + lay.xs, xl + row0 * D, ntok * rowb, &full[s]);
@@ -462,25 +503,25 @@ __global__ void __launch_bounds__(kMaxThreads, (Shape<MODE, HAS_Y>::kMinBlocks))
                 bulk_g2s(st + lay.dts + r * rowb, dtl + (row0 + r) * D + d0, rowb, &full[s]);
             }
         }
-        bulk_g2s(st + lay.bs, Bl + row0 * kN, ntok * kN * sz, &full[s]);
-        if (HAS_Y) bulk_g2s(st + lay.cs, Cl + row0 * kN, ntok * kN * sz, &full[s]);
+        bulk_g2s(st + lay.bs, Bl + row0 * kN, ntok * kN * SZ, &full[s]);
+        if (C::HAS_Y) bulk_g2s(st + lay.cs, Cl + row0 * kN, ntok * kN * SZ, &full[s]);
     };
     if (tid == 0)
         for (int64_t k = 0; k < min64(STAGES, ntiles); ++k) issue(k);
 
     // ---- initial state (overlaps the first copies) ----
-    f2 h[kCPT][8];
+    f2 h[CPT][8];
     bool h0_valid = false;
     int64_t h0_row = 0;
-    if constexpr (HAS_H0) {
+    if constexpr (C::HAS_H0) {
         h0_row = p.idx ? p.idx[chunk] : chunk;
         h0_valid = h0_row >= 0 && h0_row < p.bank_entries;
         if (!h0_valid && !(p.idx && h0_row == -1) && tid == 0)
             atomicOr(&g_scan_status, PRECOG_DEV_BAD_INDEX);
     }
 #pragma unroll
-    for (int j = 0; j < kCPT; ++j) {
-        if (HAS_H0 && h0_valid) {
+    for (int j = 0; j < CPT; ++j) {
+        if (C::HAS_H0 && h0_valid) {
             const int64_t off =
                 ((h0_row * p.L_bank + p.layer0 + layer) * static_cast<int64_t>(D) + d0 + dl + j) * kN;
             load_state16(p.bank, p.bank_dtype, off, h[j]);
@@ -490,9 +531,9 @@ __global__ void __launch_bounds__(kMaxThreads, (Shape<MODE, HAS_Y>::kMinBlocks))
         }
     }
     const unsigned wmask = __activemask();
-    float Lw[kCPT], kk[kCPT];
+    float Lw[CPT], kk[CPT];
 #pragma unroll
-    for (int j = 0; j < kCPT; ++j) {
+    for (int j = 0; j < CPT; ++j) {
         Lw[j] = 0.f;
         kk[j] = -kpow[j];
     }
@@ -500,7 +541,7 @@ __global__ void __launch_bounds__(kMaxThreads, (Shape<MODE, HAS_Y>::kMinBlocks))
     // ---- time loop ----
     void *yrow = nullptr;
     const int64_t y_stride = D;
-    if (HAS_Y) {
+    if (C::HAS_Y) {
         const int64_t off = (static_cast<int64_t>(layer) * p.T_tot + start) * D + d0 + dl;
         yrow = (p.y_dtype == PRECOG_F32) ? static_cast<void *>(static_cast<float *>(p.y) + off)
                                          : static_cast<void *>(static_cast<__nv_bfloat16 *>(p.y) + off);
@@ -509,13 +550,13 @@ __global__ void __launch_bounds__(kMaxThreads, (Shape<MODE, HAS_Y>::kMinBlocks))
         const int s = static_cast<int>(k % STAGES);
         const uint32_t par = static_cast<uint32_t>((k / STAGES) & 1);
         unsigned char *st = stage0 + s * lay.bytes;
-        const int ntok = static_cast<int>(min64(kTile, len - k * kTile));
+        const int ntok = static_cast<int>(min64(TILE, len - k * TILE));
         const bool ok = mbar_wait(&full[s], par);
-        if (CONV && ok) {
+        if (C::CONV && ok) {
             const TIn *bsrc = reinterpret_cast<const TIn *>(st + lay.bs);
             float *bdst = reinterpret_cast<float *>(st + lay.bf);
             for (int i = tid; i < ntok * kN; i += nthr) bdst[i] = to_f32(bsrc[i]);
-            if (HAS_Y) {
+            if (C::HAS_Y) {
                 const TIn *csrc = reinterpret_cast<const TIn *>(st + lay.cs);
                 float *cdst = reinterpret_cast<float *>(st + lay.cf);
                 for (int i = tid; i < ntok * kN; i += nthr) cdst[i] = to_f32(csrc[i]);
@@ -525,21 +566,20 @@ __global__ void __launch_bounds__(kMaxThreads, (Shape<MODE, HAS_Y>::kMinBlocks))
             // Give up on this chunk: record it, let issued copies land, leave.
             if (tid == 0) {
                 atomicOr(&g_scan_status, PRECOG_DEV_TIMEOUT);
-                for (int64_t kk2 = k; kk2 < min64(k + STAGES, ntiles); ++kk2)
-                    mbar_wait(&full[kk2 % STAGES], static_cast<uint32_t>((kk2 / STAGES) & 1));
+                for (int64_t k2 = k; k2 < min64(k + STAGES, ntiles); ++k2)
+                    mbar_wait(&full[k2 % STAGES], static_cast<uint32_t>((k2 / STAGES) & 1));
             }
             return;
         }
-        if constexpr (RESCALED) {
-            scan_tile_rescaled<TIn>(st, lay, DS, dl, ntok, h, Lw, kk, wmask);
+        if constexpr (C::RESCALED) {
+            scan_tile_rescaled<C>(st, lay, DS, dl, ntok, h, Lw, kk, wmask);
         } else {
-            scan_tile<TIn, HAS_Y, MODE == kPower>(st, lay, DS, dl, ntok, h, kpow, kgen, yrow,
-                                                 p.y_dtype, y_stride);
+            scan_tile_direct<C>(st, lay, DS, dl, ntok, h, kpow, kgen, yrow, p.y_dtype, y_stride);
         }
-        if (HAS_Y) {
+        if (C::HAS_Y) {
             yrow = (p.y_dtype == PRECOG_F32)
-                       ? static_cast<void *>(static_cast<float *>(yrow) + kTile * y_stride)
-                       : static_cast<void *>(static_cast<__nv_bfloat16 *>(yrow) + kTile * y_stride);
+                       ? static_cast<void *>(static_cast<float *>(yrow) + TILE * y_stride)
+                       : static_cast<void *>(static_cast<__nv_bfloat16 *>(yrow) + TILE * y_stride);
         }
         fence_proxy_async_smem();
         __syncthreads();
@@ -547,13 +587,13 @@ __global__ void __launch_bounds__(kMaxThreads, (Shape<MODE, HAS_Y>::kMinBlocks))
     }
 
     // ---- state capture ----
-    if constexpr (RESCALED) {
+    if constexpr (C::RESCALED) {
 #pragma unroll
-        for (int j = 0; j < kCPT; ++j) renormalise(h[j], Lw[j]);
+        for (int j = 0; j < CPT; ++j) renormalise(h[j], Lw[j]);
     }
     if (p.states) {
 #pragma unroll
-        for (int j = 0; j < kCPT; ++j) {
+        for (int j = 0; j < CPT; ++j) {
             const int64_t off =
                 ((chunk * p.L_out + p.layer0 + layer) * static_cast<int64_t>(D) + d0 + dl + j) * kN;
             store_state16(p.states, p.state_dtype, off, h[j]);
@@ -561,32 +601,45 @@ __global__ void __launch_bounds__(kMaxThreads, (Shape<MODE, HAS_Y>::kMinBlocks))
     }
 }
 
-int pick_slice(int D, int sz) {
+// Widest channel slice (<= kMaxSlice channels, 16-byte rows) that divides D
+// into whole threads of CPT channels.
+int pick_slice(int D, int sz, int cpt) {
     const int cands[] = {256, 128, 64, 32, 16, 8, 4, 2};
     for (int ds : cands)
-        if (D % ds == 0 && (ds * sz) % 16 == 0 && ds / kCPT <= kMaxThreads) return ds;
+        if (ds <= kMaxSlice && D % ds == 0 && (ds * sz) % 16 == 0 && ds % cpt == 0) return ds;
     return 0;
 }
 
-template <typename TIn, bool HAS_Y, bool HAS_H0, int MODE>
-cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
-    const int sz = sizeof(TIn);
-    const int DS = pick_slice(p.D, sz);
+template <class C>
+cudaError_t launch_cfg(const ScanParams &p, cudaStream_t stream) {
+    const int DS = pick_slice(p.D, C::SZ, C::CPT);
     if (DS == 0) return cudaErrorInvalidValue;
     const int slices = p.D / DS;
-    const StageLayout lay = stage_layout(DS, sz, HAS_Y, !std::is_same<TIn, float>::value);
-    const size_t smem = kBarBytes + static_cast<size_t>(Shape<MODE, HAS_Y>::kStagesUsed) * lay.bytes;
+    const StageLayout lay = stage_layout(C::TILE, DS, C::SZ, C::HAS_Y, C::CONV);
+    const size_t smem = kBarBytes + static_cast<size_t>(C::STAGES) * lay.bytes;
     const int64_t items = static_cast<int64_t>(p.n_layers) * p.n_chunks * slices;
     if (items == 0) return cudaSuccess;
     if (items > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-    auto kern = scan_kernel<TIn, HAS_Y, HAS_H0, MODE>;
+    auto kern = scan_kernel<C>;
     static int smem_set = 0;
     cudaError_t e = ensure_smem(reinterpret_cast<const void *>(kern), &smem_set, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    kern<<<static_cast<unsigned>(items), DS / kCPT, smem, stream>>>(p, DS, slices);
+    kern<<<static_cast<unsigned>(items), DS / C::CPT, smem, stream>>>(p, DS, slices);
     e = cudaGetLastError();
     if (e == cudaSuccess) count_launches(1);
     return e;
+}
+
+// Shapes: the rescaled capture kernel (the corpus-encode hot loop) and the
+// direct kernels (readout, prefill, general A).
+template <typename TIn, bool HAS_Y, bool HAS_H0, int MODE>
+cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
+    if constexpr (MODE == kPower && !HAS_Y) {
+        return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
+                              PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB>>(p, stream);
+    } else {
+        return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, 2, 16, 4, 3>>(p, stream);
+    }
 }
 
 template <typename TIn, int MODE>
