@@ -36,6 +36,9 @@ __device__ uint32_t g_scan_status;
 #define PRECOG_RESCALED_STAGES 2
 #define PRECOG_RESCALED_MINB 6
 #endif
+#ifndef PRECOG_RESCALED_GROUP
+#define PRECOG_RESCALED_GROUP 4
+#endif
 
 constexpr int kN = 16;          // state size (N) supported by the kernels
 constexpr int kMaxSlice = 256;  // channels per CTA at most
@@ -348,7 +351,7 @@ __device__ __forceinline__ void token_checked(f2 (&g)[CPT][8], float (&L)[CPT],
 // in the group (seen from the sign bits) sends the group through the per-token
 // check. One warp vote per group; the fast path then carries no branch, so the
 // power chains of the group's tokens can interleave.
-constexpr int kGroup = 4;
+constexpr int kGroup = PRECOG_RESCALED_GROUP;
 
 template <class C>
 __device__ __forceinline__ void scan_tile_rescaled(const unsigned char *st, const StageLayout &lay,
