@@ -63,6 +63,13 @@ struct RetrieveParams {
 };
 
 size_t retrieve_workspace_size(int64_t M, int32_t dim, int32_t n_queries);
+
+// Tensor-core path (retrieve_tc.cu): fp16/bf16 index, batches of queries.
+size_t retrieve_tc_smem_bytes();
+int retrieve_tc_grid(int64_t M, int sms);
+cudaError_t launch_retrieve_tc(const RetrieveParams &p, int grid, cudaStream_t stream,
+                               uint64_t *launches);
+cudaError_t retrieve_tc_status_word_read_clear(uint32_t *bits);
 cudaError_t launch_retrieve(const RetrieveParams &p, cudaStream_t stream);
 cudaError_t retrieve_status_word_read_clear(uint32_t *bits);
 

@@ -8,6 +8,7 @@
 // (score, row) pair is packed into one 64-bit key ordered by score, then by
 // lower row; per-CTA maxima go to the workspace and a finalize kernel reduces
 // them. A NaN score never enters a key, so it never wins.
+#include <algorithm>
 #include <type_traits>
 
 #include "../../include/precog.h"
@@ -212,24 +213,23 @@ cudaError_t gemv_pass_vpl(const RetrieveParams &p, int grid, int q0, cudaStream_
 }
 
 template <typename T>
-cudaError_t launch_gemv(const RetrieveParams &p, cudaStream_t stream) {
-    const int grid = gemv_grid(p.M);
-    auto *partial = static_cast<unsigned long long *>(p.workspace);
-    uint64_t launches = 0;
+cudaError_t launch_gemv(const RetrieveParams &p, cudaStream_t stream, int grid, uint64_t *launches) {
     cudaError_t e = cudaSuccess;
     if (p.n_queries == 1) {
         e = gemv_pass_vpl<T, 1>(p, grid, 0, stream);
-        ++launches;
+        ++*launches;
     } else {
-        for (int q0 = 0; q0 < p.n_queries && e == cudaSuccess; q0 += kQB, ++launches)
+        for (int q0 = 0; q0 < p.n_queries && e == cudaSuccess; q0 += kQB, ++*launches)
             e = gemv_pass_vpl<T, kQB>(p, grid, q0, stream);
     }
-    if (e != cudaSuccess) return e;
-    finalize_kernel<<<(p.n_queries + 127) / 128, 128, 0, stream>>>(partial, grid, p.n_queries,
-                                                                    p.best_idx, p.best_score);
-    e = cudaGetLastError();
-    if (e == cudaSuccess) count_launches(launches + 1);
     return e;
+}
+
+// Batches larger than one GEMV pass run on the tensor cores (16-bit keys).
+constexpr int kTcMinQueries = kQB + 1;
+
+bool use_tc(const RetrieveParams &p) {
+    return p.dtype != PRECOG_F32 && p.n_queries >= kTcMinQueries && p.M > 0;
 }
 
 }  // namespace
@@ -237,25 +237,48 @@ cudaError_t launch_gemv(const RetrieveParams &p, cudaStream_t stream) {
 size_t retrieve_workspace_size(int64_t M, int32_t dim, int32_t n_queries) {
     (void)dim;
     if (n_queries <= 0) return 0;
-    return static_cast<size_t>(gemv_grid(M)) * n_queries * sizeof(unsigned long long);
+    const int parts = std::max(gemv_grid(M), retrieve_tc_grid(M, num_sms()));
+    return static_cast<size_t>(parts) * n_queries * sizeof(unsigned long long);
 }
 
 cudaError_t launch_retrieve(const RetrieveParams &p, cudaStream_t stream) {
     if (p.n_queries == 0) return cudaSuccess;
     const int sz = p.dtype == PRECOG_F32 ? 4 : 2;
     if (p.dim * sz / 16 > kMaxVecsPerRow) return cudaErrorInvalidValue;
-    switch (p.dtype) {
-        case PRECOG_F16: return launch_gemv<__half>(p, stream);
-        case PRECOG_BF16: return launch_gemv<__nv_bfloat16>(p, stream);
-        default: return launch_gemv<float>(p, stream);
+    uint64_t launches = 0;
+    cudaError_t e;
+    int parts;
+    if (use_tc(p)) {
+        parts = retrieve_tc_grid(p.M, num_sms());
+        e = launch_retrieve_tc(p, parts, stream, &launches);
+    } else {
+        parts = gemv_grid(p.M);
+        switch (p.dtype) {
+            case PRECOG_F16: e = launch_gemv<__half>(p, stream, parts, &launches); break;
+            case PRECOG_BF16: e = launch_gemv<__nv_bfloat16>(p, stream, parts, &launches); break;
+            default: e = launch_gemv<float>(p, stream, parts, &launches); break;
+        }
     }
+    if (e == cudaSuccess) {
+        finalize_kernel<<<(p.n_queries + 127) / 128, 128, 0, stream>>>(
+            static_cast<const unsigned long long *>(p.workspace), parts, p.n_queries, p.best_idx,
+            p.best_score);
+        e = cudaGetLastError();
+        if (e == cudaSuccess) ++launches;
+    }
+    count_launches(launches);
+    return e;
 }
 
 cudaError_t retrieve_status_word_read_clear(uint32_t *bits) {
-    uint32_t zero = 0;
+    uint32_t zero = 0, tc = 0;
     cudaError_t e = cudaMemcpyFromSymbol(bits, g_retrieve_status, sizeof(uint32_t));
     if (e != cudaSuccess) return e;
-    return cudaMemcpyToSymbol(g_retrieve_status, &zero, sizeof(uint32_t));
+    e = cudaMemcpyToSymbol(g_retrieve_status, &zero, sizeof(uint32_t));
+    if (e != cudaSuccess) return e;
+    e = retrieve_tc_status_word_read_clear(&tc);
+    *bits |= tc;
+    return e;
 }
 
 }  // namespace precog

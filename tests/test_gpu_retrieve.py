@@ -124,3 +124,44 @@ def test_query_workload_full_index(cuda_device, Q):
         assert idx[qi] == bi and abs(score[qi] - bs) < 1e-5
     del index
     torch.cuda.empty_cache()
+
+
+# ------------------------------------------------------------- tensor-core path (Q >= 5)
+
+
+@pytest.mark.parametrize("dtype_name", ["float16", "bfloat16"])
+@pytest.mark.parametrize("M,Q,dim", [(1, 5, 64), (127, 9, 64), (128, 130, 96), (129, 256, 768),
+                                     (4099, 300, 96), (20000, 17, 136)])
+def test_tensor_core_exact_integer_scores(cuda_device, dtype_name, M, Q, dim):
+    """Batches of five or more queries over a 16-bit index take the tcgen05 path. Small
+    integer keys and queries make every score exact in fp32, so indices and scores must
+    equal the oracle's bit for bit: ragged tiles (M), ragged and multi-pass query batches
+    (Q > 128, Q > 256), a K tail (dim not a multiple of 64), many exact ties."""
+    import torch
+    dtype = getattr(torch, dtype_name)
+    rng = np.random.default_rng(M * 31 + Q * 7 + dim)
+    index = rng.integers(-3, 4, size=(M, dim)).astype(np.float32)
+    queries = rng.integers(-3, 4, size=(Q, dim)).astype(np.float32)
+    idx, score = _run(torch.from_numpy(index).to(cuda_device, dtype),
+                      torch.from_numpy(queries).to(cuda_device, dtype))
+    ref_i, ref_s = oracle.retrieve(index, queries)
+    np.testing.assert_array_equal(idx, ref_i)
+    np.testing.assert_array_equal(score.astype(np.float64), ref_s)
+
+
+def test_tensor_core_ties_and_nan_rows(cuda_device):
+    """The tcgen05 path keeps the lowest row among equal best scores even when they sit
+    in different tiles and CTAs, and never lets a NaN row win."""
+    import torch
+    rng = np.random.default_rng(5)
+    M, dim, Q = 300_000, 768, 16
+    index = (rng.standard_normal((M, dim)) * 0.01).astype(np.float16)
+    best = rng.standard_normal((Q, dim)).astype(np.float16)
+    planted = [(q, r) for q in range(Q) for r in (290_001 - 97 * q, 150_000 + 13 * q, 17 * q + 3)]
+    for q, r in planted:
+        index[r] = best[q]
+    index[[1, 2, 299_999]] = np.nan
+    idx, score = _run(torch.from_numpy(index).to(cuda_device), torch.from_numpy(best).to(cuda_device))
+    for q in range(Q):
+        assert idx[q] == min(r for qq, r in planted if qq == q)
+    assert np.all(np.isfinite(score))
