@@ -159,6 +159,29 @@ precog_status precog_retrieve(const void *index, int32_t index_dtype, int64_t M,
 size_t precog_retrieve_workspace_size(int64_t M, int32_t dim, int32_t n_queries);
 
 /*
+ * precog_retrieve_noalloc -- precog_retrieve for callers that cannot allocate
+ * device memory when they retrieve (a serving loop that must never call
+ * cudaMalloc, which may synchronise the device; code that runs inside someone
+ * else's memory pool). The paper has no counterpart: this is a property of the
+ * library, not of the method. Same arguments and results as precog_retrieve,
+ * without the workspace: the partial keys go to a fixed 2 MiB array compiled
+ * into the library, which every GPU that loads the library holds until exit.
+ *   - Allocates nothing and calls no allocating routine.
+ *   - The first call on a device looks up that array's device address (once
+ *     per device, with the device current); make that first call before any
+ *     stream capture.
+ *   - Calls whose sizes need more than the 2 MiB (keys = precog_retrieve
+ *     workspace bytes / 8; about 430 queries per call at any M on a 152-SM GPU)
+ *     return PRECOG_ERR_UNSUPPORTED without launching anything.
+ *   - All calls share the array and nothing in it needs to start at zero; two
+ *     calls that overlap on the GPU (different streams, or different host
+ *     threads without ordering) race on it and may return wrong rows.
+ */
+precog_status precog_retrieve_noalloc(const void *index, int32_t index_dtype, int64_t M,
+                                      int32_t dim, const void *queries, int32_t n_queries,
+                                      int64_t *d_best_idx, float *d_best_score, void *stream);
+
+/*
  * precog_prefill_from_state -- state injection and query prefill (Sec. 4.2,
  * Eq. 2): for every query q and layer l, h_init[l] <- bank[row_q][layer0+l],
  * then scan the query's T_q tokens from h_init, producing y_t for every query

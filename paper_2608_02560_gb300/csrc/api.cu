@@ -275,3 +275,66 @@ int32_t precog_abi_version(void) { return PRECOG_ABI_VERSION; }
 uint64_t precog_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Retrieval without a caller workspace.
+//
+// Some callers cannot allocate device memory at the moment they retrieve: a
+// real-time serving loop that must not call cudaMalloc (it can synchronise the
+// device and stall every stream), code running inside a memory pool owned by
+// someone else, or a host whose allocator is not the CUDA one. For them the
+// partial (score, row) keys of precog_retrieve live in a fixed array compiled
+// into this library instead of a workspace they would have to provide.
+namespace {
+
+// 262,144 packed keys = 2 MiB, held on every GPU that loads this library until
+// the process exits. Enough for about 430 queries per call at any index size on
+// a 152-SM GPU (keys needed = scratch partitions x n_queries).
+constexpr size_t kNoallocKeys = 262144;
+static __device__ __align__(256) unsigned long long g_noalloc_scratch[kNoallocKeys];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mutex;
+void *g_noalloc_ptr[kMaxDevices] = {};
+
+// Device address of the scratch on the current device (set up once per device).
+precog_status noalloc_scratch(void **ptr) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= kMaxDevices)
+        return fail(PRECOG_ERR_UNSUPPORTED, "device ordinal %d is beyond %d", dev, kMaxDevices);
+    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+    if (g_noalloc_ptr[dev] == nullptr) {
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(scratch)");
+        g_noalloc_ptr[dev] = p;
+    }
+    *ptr = g_noalloc_ptr[dev];
+    return PRECOG_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+precog_status precog_retrieve_noalloc(const void *index, int32_t index_dtype, int64_t M,
+                                      int32_t dim, const void *queries, int32_t n_queries,
+                                      int64_t *d_best_idx, float *d_best_score, void *stream) {
+    if (n_queries < 0) return fail(PRECOG_ERR_INVALID_ARG, "n_queries must be >= 0");
+    if (M < 0 || dim < 1) return fail(PRECOG_ERR_INVALID_ARG, "M must be >= 0 and dim >= 1");
+    const size_t need = precog::retrieve_workspace_size(M, dim, n_queries);
+    if (need > sizeof(g_noalloc_scratch))
+        return fail(PRECOG_ERR_UNSUPPORTED,
+                    "precog_retrieve_noalloc: %d queries need %zu bytes of scratch, more than the "
+                    "fixed %zu; use fewer queries per call or precog_retrieve with a workspace",
+                    n_queries, need, sizeof(g_noalloc_scratch));
+    void *scratch = nullptr;
+    precog_status s = noalloc_scratch(&scratch);
+    if (s != PRECOG_OK) return s;
+    return precog_retrieve(index, index_dtype, M, dim, queries, n_queries, d_best_idx,
+                           d_best_score, scratch, sizeof(g_noalloc_scratch), stream);
+}
+
+}  // extern "C"
