@@ -36,6 +36,13 @@ __device__ uint32_t g_scan_status;
 #define PRECOG_RESCALED_STAGES 2
 #define PRECOG_RESCALED_MINB 6
 #endif
+// Shape of the direct-update kernels with A stated structured (readout, prefill).
+#ifndef PRECOG_DIRECT_CPT
+#define PRECOG_DIRECT_CPT 4
+#define PRECOG_DIRECT_TILE 16
+#define PRECOG_DIRECT_STAGES 2
+#define PRECOG_DIRECT_MINB 6
+#endif
 #ifndef PRECOG_RESCALED_GROUP
 #define PRECOG_RESCALED_GROUP 4
 #endif
@@ -641,7 +648,13 @@ cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
         return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
                               PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB>>(p, stream);
     } else {
-        return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, 2, 16, 4, 3>>(p, stream);
+        if constexpr (MODE == kPower) {
+            return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, PRECOG_DIRECT_CPT, PRECOG_DIRECT_TILE,
+                                  PRECOG_DIRECT_STAGES, PRECOG_DIRECT_MINB>>(p, stream);
+        } else {
+            // general A keeps 16 exponent coefficients per channel: 2 channels per thread
+            return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, 2, 16, 4, 3>>(p, stream);
+        }
     }
 }
 
