@@ -32,15 +32,27 @@ __device__ uint32_t g_scan_status;
 // stages, resident blocks per SM for the register budget).
 #ifndef PRECOG_RESCALED_CPT
 #define PRECOG_RESCALED_CPT 4
+#endif
+#ifndef PRECOG_RESCALED_TILE
 #define PRECOG_RESCALED_TILE 16
+#endif
+#ifndef PRECOG_RESCALED_STAGES
 #define PRECOG_RESCALED_STAGES 2
+#endif
+#ifndef PRECOG_RESCALED_MINB
 #define PRECOG_RESCALED_MINB 6
 #endif
 // Shape of the direct-update kernels with A stated structured (readout, prefill).
 #ifndef PRECOG_DIRECT_CPT
 #define PRECOG_DIRECT_CPT 4
+#endif
+#ifndef PRECOG_DIRECT_TILE
 #define PRECOG_DIRECT_TILE 16
+#endif
+#ifndef PRECOG_DIRECT_STAGES
 #define PRECOG_DIRECT_STAGES 2
+#endif
+#ifndef PRECOG_DIRECT_MINB
 #define PRECOG_DIRECT_MINB 6
 #endif
 #ifndef PRECOG_RESCALED_GROUP
