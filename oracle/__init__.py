@@ -13,6 +13,10 @@ module compiles it with gcc and marshals numpy arrays into it.
 * :func:`retrieve` -- exact top-1 dot-product retrieval (Sec. 4.2), lowest row
   on ties, NaN never wins.
 * :func:`rollout` -- one chunk convenience wrapper of :func:`scan`.
+* :func:`retrieve_topk` -- the k best rows per query by exact score (ties to the
+  lower row), the top-k of Sec. 4.2 / Sec. 5.4.
+* :func:`compose` -- the softmax-weighted state composition of Sec. 4.4
+  (multi-chunk extension) and Eq. smc-fusion.
 """
 from __future__ import annotations
 
@@ -58,6 +62,9 @@ def _load():
         lib.oracle_scan.restype = ctypes.c_int
         lib.oracle_scan.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, p_i64,
                                     p_f64, p_f64, p_f64, p_f64, p_f64, p_f64, p_f64, p_f64]
+        lib.oracle_scores.restype = ctypes.c_int
+        lib.oracle_scores.argtypes = [ctypes.c_int64, ctypes.c_int64, p_f64, ctypes.c_int64, p_f64,
+                                      p_f64]
         lib.oracle_retrieve.restype = ctypes.c_int
         lib.oracle_retrieve.argtypes = [ctypes.c_int64, ctypes.c_int64, p_f64, ctypes.c_int64,
                                         p_f64, p_i64, p_f64]
@@ -140,3 +147,56 @@ def retrieve(index, queries):
     if rc != 0:
         raise ValueError(f"oracle_retrieve rejected its arguments (rc={rc})")
     return best_idx, best_score
+
+
+def scores(index, queries):
+    """All dot products ``[Q, M]`` in double."""
+    lib = _load()
+    index = _f64(index)
+    queries = _f64(queries)
+    if queries.ndim == 1:
+        queries = queries.reshape(1, -1)
+    M, dim = index.shape
+    Q = queries.shape[0]
+    out = np.empty((Q, M), dtype=np.float64)
+    rc = lib.oracle_scores(M, dim, _ptr(index, ctypes.c_double), Q, _ptr(queries, ctypes.c_double),
+                           _ptr(out, ctypes.c_double))
+    if rc != 0:
+        raise ValueError(f"oracle_scores rejected its arguments (rc={rc})")
+    return out
+
+
+def retrieve_topk(index, queries, k):
+    """The k rows with the highest exact score per query, best first; among equal scores
+    the lower row comes first; NaN scores are never selected; missing entries are row -1
+    with score NaN. Returns ``(rows int64 [Q, k], scores float64 [Q, k])``."""
+    S = scores(index, queries)
+    Q, M = S.shape
+    rows = np.full((Q, k), -1, dtype=np.int64)
+    vals = np.full((Q, k), np.nan)
+    for q in range(Q):
+        cand = [(-S[q, i], i) for i in range(M) if not np.isnan(S[q, i])]
+        cand.sort()
+        for j, (neg, i) in enumerate(cand[:k]):
+            rows[q, j] = i
+            vals[q, j] = -neg
+    return rows, vals
+
+
+def compose(bank_rows, row_scores, temperature=1.0):
+    """h_init = sum_j w_j h^(j), w = softmax(score / temperature) over the valid entries
+    (Sec. 4.4, Eq. smc-fusion). ``bank_rows [k, ...]`` are the states of the k retrieved
+    chunks, ``row_scores [k]`` their scores (NaN marks a missing entry, weight 0)."""
+    s = np.asarray(row_scores, dtype=np.float64)
+    valid = ~np.isnan(s)
+    out = np.zeros(np.asarray(bank_rows).shape[1:], dtype=np.float64)
+    if not valid.any():
+        return out
+    z = s[valid] / temperature
+    e = np.exp(z - z.max())
+    w = e / e.sum()
+    rows = np.asarray(bank_rows, dtype=np.float64)[valid]
+    for j in range(len(w)):
+        out = out + w[j] * rows[j]
+    return out
+

@@ -128,3 +128,24 @@ int oracle_retrieve(int64_t M, int64_t dim, const double *index, int64_t Q,
     }
     return ORACLE_OK;
 }
+
+/*
+ * oracle_scores: every dot product <query_q, key_i> in double (Sec. 4.2;
+ * the scores that top-1 and top-k retrieval rank).
+ *   scores [Q][M]
+ */
+int oracle_scores(int64_t M, int64_t dim, const double *index, int64_t Q,
+                  const double *queries, double *scores)
+{
+    if (M < 0 || dim <= 0 || Q < 0 || scores == NULL)
+        return ORACLE_BAD_ARG;
+    for (int64_t q = 0; q < Q; ++q)
+        for (int64_t i = 0; i < M; ++i) {
+            double s = 0.0;
+            for (int64_t k = 0; k < dim; ++k)
+                s += queries[q * dim + k] * index[i * dim + k];
+            scores[q * M + i] = s;
+        }
+    return ORACLE_OK;
+}
+

@@ -297,3 +297,64 @@ def test_bf16_storage_tolerance_helper():
     bumped = stored.copy()
     bumped[np.argmax(np.abs(ref))] *= 1 + 2.0 ** -6         # two ulps off at the maximum
     assert rel_err_stored(bumped, ref) > 2e-3
+
+
+# ---------------------------------------------------------------- top-k and composition
+
+
+def test_topk_matches_numpy_stable_argsort():
+    """Top-k = the first k of a stable sort by descending exact score (lower row first
+    among equals), checked with numpy's stable argsort on exact small-integer scores."""
+    rng = np.random.default_rng(3)
+    M, dim, Q, k = 200, 9, 6, 5
+    index = rng.integers(-2, 3, size=(M, dim)).astype(float)
+    queries = rng.integers(-2, 3, size=(Q, dim)).astype(float)
+    rows, vals = oracle.retrieve_topk(index, queries, k)
+    S = queries @ index.T
+    for q in range(Q):
+        order = np.argsort(-S[q], kind="stable")[:k]
+        np.testing.assert_array_equal(rows[q], order)
+        np.testing.assert_array_equal(vals[q], S[q, order])
+    r1, s1 = oracle.retrieve(index, queries)
+    np.testing.assert_array_equal(rows[:, 0], r1)          # k = 1 is top-1 retrieval
+
+
+def test_topk_nan_and_short_index():
+    index = np.array([[1.0, 0.0], [np.nan, 1.0], [0.5, 0.0]])
+    rows, vals = oracle.retrieve_topk(index, np.array([[1.0, 1.0]]), 4)
+    assert list(rows[0]) == [0, 2, -1, -1]
+    assert vals[0, 0] == 1.0 and vals[0, 1] == 0.5 and np.isnan(vals[0, 2:]).all()
+
+
+def test_compose_softmax_weights():
+    """Weights are the textbook softmax (scipy) of score / temperature; equal scores give
+    the plain average; one entry gives that entry; missing entries get no weight."""
+    scipy_special = pytest.importorskip("scipy.special")
+    rng = np.random.default_rng(8)
+    rows = rng.standard_normal((3, 4, 5))
+    sc = np.array([0.9, 0.2, -0.3])
+    for tau in (1.0, 0.1):
+        w = scipy_special.softmax(sc / tau)
+        np.testing.assert_allclose(oracle.compose(rows, sc, tau),
+                                   np.tensordot(w, rows, axes=1), rtol=1e-13, atol=1e-13)
+    np.testing.assert_allclose(oracle.compose(rows, np.full(3, 0.4)), rows.mean(axis=0), rtol=1e-13)
+    np.testing.assert_array_equal(oracle.compose(rows[:1], [0.7]), rows[0])
+    np.testing.assert_allclose(oracle.compose(rows, [0.5, np.nan, 0.5]), (rows[0] + rows[2]) / 2,
+                               rtol=1e-13)
+
+
+def test_composition_commutes_with_the_scan():
+    """The scan is affine in its initial state (Eq. unroll): with weights summing to one,
+    S(sum_j w_j h_j, q) = sum_j w_j S(h_j, q) -- injecting the composed state equals
+    composing the individually injected rollouts."""
+    D, N, T = 3, 4, 20
+    x, dt, A, B, C = _rand_inputs(T, D, N, seed=17)
+    rng = np.random.default_rng(4)
+    hs = rng.standard_normal((3, D, N))
+    sc = np.array([0.3, 0.8, 0.1])
+    h_comp, y_comp = oracle.rollout(x, dt, A, B, C, h0=oracle.compose(hs, sc), want_y=True)
+    e = np.exp(sc - sc.max())
+    w = e / e.sum()
+    parts = [oracle.rollout(x, dt, A, B, C, h0=hs[j], want_y=True) for j in range(3)]
+    np.testing.assert_allclose(h_comp, sum(w[j] * parts[j][0] for j in range(3)), rtol=1e-11, atol=1e-12)
+    np.testing.assert_allclose(y_comp, sum(w[j] * parts[j][1] for j in range(3)), rtol=1e-11, atol=1e-12)
