@@ -210,6 +210,47 @@ precog_status precog_prefill_from_state(const precog_scan_inputs *in, int32_t n_
                                         void *state_out, int32_t state_dtype, void *stream);
 
 /*
+ * precog_retrieve_topk -- the k best rows per query (1 <= k <= 8), best first:
+ * the top-k retrieval of Sec. 4.2 (k = 3 by default in the paper) that feeds
+ * the softmax-weighted composition of Sec. 4.4 and Eq. smc-fusion. Same
+ * scoring and tie rule as precog_retrieve (ties to the lower row, NaN never
+ * selected); missing entries (fewer than k comparable rows) are row -1 with
+ * score NaN.
+ *   d_idx    device int64 [n_queries][k] (written)
+ *   d_score  device fp32 [n_queries][k] (written), or NULL
+ *   workspace at least precog_retrieve_topk_workspace_size(M, dim, n_queries)
+ */
+precog_status precog_retrieve_topk(const void *index, int32_t index_dtype, int64_t M, int32_t dim,
+                                   const void *queries, int32_t n_queries, int32_t k,
+                                   int64_t *d_idx, float *d_score, void *workspace,
+                                   size_t workspace_bytes, void *stream);
+
+/* Bytes of device workspace precog_retrieve_topk needs for these sizes (any k). */
+size_t precog_retrieve_topk_workspace_size(int64_t M, int32_t dim, int32_t n_queries);
+
+/*
+ * precog_prefill_composed -- top-k state composition, then prefill: the
+ * heuristic multi-chunk extension of Sec. 4.4 (Eq. smc-fusion),
+ *   h_init[l] = sum_j w_j bank[row_qj][layer0+l],  w = softmax(score_qj / temperature),
+ * over the valid entries of query q (a row of -1 or a NaN score has weight 0;
+ * a row outside the bank has weight 0 and flags PRECOG_DEV_BAD_INDEX), then
+ * the same prefill as precog_prefill_from_state. Weights and the sum are fp32.
+ * Unlike top-1 injection this is not exact in-context equivalence (Theorem 1
+ * covers a single chunk only).
+ *   k          1..8 entries per query; k == 1 is precog_prefill_from_state
+ *   d_idx      device int64 [n_queries][k] rows (e.g. precog_retrieve_topk's)
+ *   d_score    device fp32 [n_queries][k] scores (ignored when k == 1)
+ *   temperature > 0; the paper's plain softmax of the similarity is 1.0
+ * Other arguments as precog_prefill_from_state.
+ */
+precog_status precog_prefill_composed(const precog_scan_inputs *in, int32_t n_queries, int32_t T_q,
+                                      const void *bank, int32_t bank_dtype, int64_t bank_entries,
+                                      int32_t L_bank, int32_t layer0, int32_t k,
+                                      const int64_t *d_idx, const float *d_score, float temperature,
+                                      void *y_out, int32_t y_dtype, void *state_out,
+                                      int32_t state_dtype, void *stream);
+
+/*
  * precog_device_status -- synchronise `stream`, then report and clear the
  * device status word shared by all calls on this device. *bits_out receives
  * the PRECOG_DEV_* bits seen since the last clear. Returns PRECOG_OK when no

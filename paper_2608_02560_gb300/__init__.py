@@ -11,6 +11,8 @@ Functions carry the C names:
 * :func:`precog_encode_chunks`    -- offline indexing (Sec. 4.2)
 * :func:`precog_retrieve`         -- exact top-1 retrieval (Sec. 4.2)
 * :func:`precog_prefill_from_state` -- injection (Eq. 2) + query prefill
+* :func:`precog_retrieve_topk`    -- top-k retrieval (Sec. 4.2 / 5.4)
+* :func:`precog_prefill_composed` -- softmax-weighted top-k injection (Sec. 4.4) + prefill
 * :func:`precog_device_status`    -- device-side status word
 """
 from __future__ import annotations
@@ -68,6 +70,13 @@ def load_library(path: str = LIB_PATH):
     lib.precog_prefill_from_state.restype = i32
     lib.precog_prefill_from_state.argtypes = [ctypes.POINTER(ScanInputs), i32, i32, vp, i32, i64,
                                               i32, i32, vp, vp, i32, vp, i32, vp]
+    lib.precog_retrieve_topk.restype = i32
+    lib.precog_retrieve_topk.argtypes = [vp, i32, i64, i32, vp, i32, i32, vp, vp, vp, sz, vp]
+    lib.precog_retrieve_topk_workspace_size.restype = sz
+    lib.precog_retrieve_topk_workspace_size.argtypes = [i64, i32, i32]
+    lib.precog_prefill_composed.restype = i32
+    lib.precog_prefill_composed.argtypes = [ctypes.POINTER(ScanInputs), i32, i32, vp, i32, i64, i32,
+                                            i32, i32, vp, vp, ctypes.c_float, vp, i32, vp, i32, vp]
     lib.precog_device_status.restype = i32
     lib.precog_device_status.argtypes = [vp, ctypes.POINTER(ctypes.c_uint32)]
     lib.precog_status_string.restype = ctypes.c_char_p
@@ -131,6 +140,8 @@ def scan_inputs(x, dt, B, A, C=None, a_kind: int = PRECOG_A_GENERAL) -> ScanInpu
     if A.shape != (L, D, N) or A.dtype != torch.float32:
         raise ValueError("A must be float32 [L, D, N]")
     s = ScanInputs()
+    # the struct holds raw device pointers: keep the tensors alive as long as it lives
+    s._keepalive = (x, dt, B, C, A)
     s.n_layers, s.D, s.N = L, D, N
     s.in_dtype = _dtype_code(x)
     s.a_kind = a_kind
@@ -187,6 +198,34 @@ def precog_prefill_from_state(inputs: ScanInputs, n_queries: int, T_q: int, bank
         layer0, _ptr(idx), _ptr(y_out), _dtype_code(y_out) if y_out is not None else PRECOG_F32,
         _ptr(state_out), _dtype_code(state_out) if state_out is not None else PRECOG_F32,
         _stream(stream)))
+
+
+def precog_retrieve_topk(index, queries, k, best_idx, best_score=None, workspace=None, stream=None):
+    """The k best rows per query into ``best_idx [Q, k]`` (int64) and ``best_score [Q, k]``."""
+    import torch
+    lib = load_library()
+    M, dim = index.shape
+    Q = queries.shape[0]
+    need = int(lib.precog_retrieve_topk_workspace_size(M, dim, Q))
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=index.device)
+    _check(lib.precog_retrieve_topk(
+        _ptr(index), _dtype_code(index), M, dim, _ptr(queries), Q, k, _ptr(best_idx),
+        _ptr(best_score), _ptr(workspace), workspace.numel() * workspace.element_size(),
+        _stream(stream)))
+
+
+def precog_prefill_composed(inputs: ScanInputs, n_queries: int, T_q: int, bank, idx, scores, k: int,
+                            temperature: float = 1.0, layer0: int = 0, y_out=None, state_out=None,
+                            stream=None):
+    """Inject sum_j softmax(scores/temperature)_j bank[idx[q, j]] and prefill each query."""
+    lib = load_library()
+    entries, L_bank = bank.shape[0], bank.shape[1]
+    _check(lib.precog_prefill_composed(
+        ctypes.byref(inputs), n_queries, T_q, _ptr(bank), _dtype_code(bank), entries, L_bank, layer0,
+        k, _ptr(idx), _ptr(scores), temperature, _ptr(y_out),
+        _dtype_code(y_out) if y_out is not None else PRECOG_F32, _ptr(state_out),
+        _dtype_code(state_out) if state_out is not None else PRECOG_F32, _stream(stream)))
 
 
 def precog_device_status(stream=None):

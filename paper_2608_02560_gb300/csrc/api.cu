@@ -196,6 +196,102 @@ precog_status precog_prefill_from_state(const precog_scan_inputs *in, int32_t n_
     return ok();
 }
 
+precog_status precog_prefill_composed(const precog_scan_inputs *in, int32_t n_queries, int32_t T_q,
+                                     const void *bank, int32_t bank_dtype, int64_t bank_entries,
+                                     int32_t L_bank, int32_t layer0, int32_t k,
+                                     const int64_t *d_idx, const float *d_score, float temperature,
+                                     void *y_out, int32_t y_dtype, void *state_out,
+                                     int32_t state_dtype, void *stream) {
+    if (k < 1 || k > 8) return fail(PRECOG_ERR_UNSUPPORTED, "k must be in [1, 8]");
+    if (d_idx == nullptr) return fail(PRECOG_ERR_INVALID_ARG, "d_idx is NULL");
+    if (k > 1 && d_score == nullptr) return fail(PRECOG_ERR_INVALID_ARG, "d_score is NULL");
+    if (!(temperature > 0.f)) return fail(PRECOG_ERR_INVALID_ARG, "temperature must be > 0");
+    if (k == 1)
+        return precog_prefill_from_state(in, n_queries, T_q, bank, bank_dtype, bank_entries, L_bank,
+                                         layer0, d_idx, y_out, y_dtype, state_out, state_dtype, stream);
+    if (n_queries < 0 || T_q < 0) return fail(PRECOG_ERR_INVALID_ARG, "n_queries and T_q must be >= 0");
+    const int64_t rows = static_cast<int64_t>(n_queries) * T_q;
+    precog_status s = check_scan_inputs(in, rows, y_out != nullptr);
+    if (s != PRECOG_OK) return s;
+    if (bank == nullptr || !state_dtype_ok(bank_dtype) || !aligned16(bank))
+        return fail(PRECOG_ERR_INVALID_ARG, "bank must be a 16-byte aligned F32 or BF16 array");
+    if (bank_entries < 0) return fail(PRECOG_ERR_INVALID_ARG, "bank_entries must be >= 0");
+    if (L_bank < 1 || layer0 < 0 || layer0 + in->n_layers > L_bank)
+        return fail(PRECOG_ERR_INVALID_ARG, "layers [layer0, layer0+n_layers) exceed L_bank");
+    if (y_out == nullptr && state_out == nullptr)
+        return fail(PRECOG_ERR_INVALID_ARG, "y_out and state_out are both NULL: nothing to do");
+    if (y_out && (!state_dtype_ok(y_dtype) || !aligned16(y_out)))
+        return fail(PRECOG_ERR_INVALID_ARG, "y_out must be 16-byte aligned F32 or BF16");
+    if (state_out && (!state_dtype_ok(state_dtype) || !aligned16(state_out)))
+        return fail(PRECOG_ERR_INVALID_ARG, "state_out must be 16-byte aligned F32 or BF16");
+    if (n_queries == 0) return ok();
+    precog::ScanParams p = base_params(in, rows);
+    p.n_chunks = n_queries;
+    p.use_fixed = 1;
+    p.fixed_len = T_q;
+    p.bank = bank;
+    p.bank_dtype = bank_dtype;
+    p.bank_entries = bank_entries;
+    p.idx = d_idx;
+    p.topk = k;
+    p.topk_scores = d_score;
+    p.inv_temp = 1.f / temperature;
+    p.L_bank = L_bank;
+    p.states = state_out;
+    p.state_dtype = state_dtype;
+    p.L_out = L_bank;
+    p.layer0 = layer0;
+    p.y = y_out;
+    p.y_dtype = y_dtype;
+    cudaError_t e = precog::launch_scan(p, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "composed prefill launch");
+    return ok();
+}
+
+size_t precog_retrieve_topk_workspace_size(int64_t M, int32_t dim, int32_t n_queries) {
+    if (M < 0 || dim < 1 || n_queries < 0) return 0;
+    return precog::retrieve_topk_workspace_size(M, dim, n_queries);
+}
+
+precog_status precog_retrieve_topk(const void *index, int32_t index_dtype, int64_t M, int32_t dim,
+                                   const void *queries, int32_t n_queries, int32_t k,
+                                   int64_t *d_idx, float *d_score, void *workspace,
+                                   size_t workspace_bytes, void *stream) {
+    if (k < 1 || k > 8) return fail(PRECOG_ERR_UNSUPPORTED, "k must be in [1, 8]");
+    const int sz = dtype_size(index_dtype);
+    if (sz == 0) return fail(PRECOG_ERR_UNSUPPORTED, "index_dtype must be F16, BF16 or F32");
+    if (M < 0) return fail(PRECOG_ERR_INVALID_ARG, "M must be >= 0");
+    if (M >= 0x7fffffffLL) return fail(PRECOG_ERR_UNSUPPORTED, "M must be below 2^31-1");
+    if (dim < 1) return fail(PRECOG_ERR_INVALID_ARG, "dim must be >= 1");
+    if ((static_cast<int64_t>(dim) * sz) % 16 != 0)
+        return fail(PRECOG_ERR_UNSUPPORTED, "dim*sizeof(dtype) must be a multiple of 16");
+    if (static_cast<int64_t>(dim) * sz > 8192)
+        return fail(PRECOG_ERR_UNSUPPORTED, "rows longer than 8 KiB (dim*sizeof(dtype)) are not implemented");
+    if (n_queries < 0) return fail(PRECOG_ERR_INVALID_ARG, "n_queries must be >= 0");
+    if (n_queries == 0) return ok();
+    if ((M > 0 && index == nullptr) || queries == nullptr || d_idx == nullptr)
+        return fail(PRECOG_ERR_INVALID_ARG, "index, queries and d_idx must be non-NULL");
+    if ((index && !aligned16(index)) || !aligned16(queries))
+        return fail(PRECOG_ERR_INVALID_ARG, "index and queries must be 16-byte aligned");
+    const size_t need = precog::retrieve_topk_workspace_size(M, dim, n_queries);
+    if (workspace_bytes < need || (need > 0 && (workspace == nullptr || !aligned16(workspace))))
+        return fail(PRECOG_ERR_INVALID_ARG, "workspace too small or misaligned (%zu bytes needed)", need);
+    precog::RetrieveParams p;
+    p.index = index;
+    p.dtype = index_dtype;
+    p.M = M;
+    p.dim = dim;
+    p.queries = queries;
+    p.n_queries = n_queries;
+    p.best_idx = d_idx;
+    p.best_score = d_score;
+    p.workspace = workspace;
+    p.workspace_bytes = workspace_bytes;
+    cudaError_t e = precog::launch_retrieve_topk(p, k, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "top-k retrieve launch");
+    return ok();
+}
+
 size_t precog_retrieve_workspace_size(int64_t M, int32_t dim, int32_t n_queries) {
     if (M < 0 || dim < 1 || n_queries < 0) return 0;
     return precog::retrieve_workspace_size(M, dim, n_queries);

@@ -28,7 +28,10 @@ struct ScanParams {
     const void *bank;
     int32_t bank_dtype;
     int64_t bank_entries;
-    const int64_t *idx;       // nullptr -> row = chunk
+    const int64_t *idx;       // nullptr -> row = chunk; [n_chunks][topk] when topk > 1
+    int32_t topk;             // rows composed per chunk (<= 1: plain injection)
+    const float *topk_scores; // [n_chunks][topk] retrieval scores (topk > 1)
+    float inv_temp;           // 1 / softmax temperature
     int32_t L_bank;           // layers per bank entry
     // outputs
     void *states;             // [n_chunks][L_out][D][N] or nullptr
@@ -70,6 +73,12 @@ int retrieve_tc_grid(int64_t M, int sms);
 cudaError_t launch_retrieve_tc(const RetrieveParams &p, int grid, cudaStream_t stream,
                                uint64_t *launches);
 cudaError_t retrieve_tc_status_word_read_clear(uint32_t *bits);
+
+// Top-k retrieval (k <= 8): partial lists of 8 packed keys per (part, query).
+size_t retrieve_topk_workspace_size(int64_t M, int32_t dim, int32_t n_queries);
+cudaError_t launch_retrieve_topk(const RetrieveParams &p, int k, cudaStream_t stream);
+cudaError_t launch_retrieve_tc_topk(const RetrieveParams &p, int grid, cudaStream_t stream,
+                                    uint64_t *launches);
 cudaError_t launch_retrieve(const RetrieveParams &p, cudaStream_t stream);
 cudaError_t retrieve_status_word_read_clear(uint32_t *bits);
 

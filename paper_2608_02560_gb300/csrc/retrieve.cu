@@ -171,6 +171,125 @@ __global__ void finalize_kernel(const unsigned long long *__restrict__ partial, 
     }
 }
 
+// ---------------------------------------------------------------------------
+// Top-k (k <= kListK) for one query per pass: every warp keeps the kListK best
+// packed keys seen so far as a sorted list, held identically by all lanes (the
+// butterfly leaves the row's score in every lane), so a row costs one compare
+// against the list's last entry unless it enters the list. The warps' lists
+// are merged per CTA in shared memory; partial[(cta * Q + q) * kListK + j].
+constexpr int kListK = 8;
+
+__device__ __forceinline__ void list_insert(unsigned long long (&l)[kListK], unsigned long long v) {
+    if (v <= l[kListK - 1]) return;
+#pragma unroll
+    for (int j = kListK - 1; j > 0; --j) {
+        // shift entries below v down by one; v lands in its sorted slot
+        const bool shift = v > l[j - 1];
+        l[j] = shift ? l[j - 1] : (v > l[j] ? v : l[j]);
+    }
+    l[0] = v > l[0] ? v : l[0];
+}
+
+template <typename T, int VPL>
+__global__ void __launch_bounds__(kThreads)
+    gemv_topk_kernel(const T *__restrict__ index, int64_t M, int dim, const T *__restrict__ queries,
+                     int n_queries, int q, unsigned long long *__restrict__ partial) {
+    constexpr int V = Vec<T>::n;
+    constexpr int RIF = 4;
+    __shared__ unsigned long long lists[kWarps][kListK];
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    const int vecs = dim / V;
+    float qv[VPL][V];
+#pragma unroll
+    for (int j = 0; j < VPL; ++j) {
+        const int v = lane + 32 * j;
+        if (v < vecs) {
+            const uint4 raw = __ldg(reinterpret_cast<const uint4 *>(queries + static_cast<int64_t>(q) * dim) + v);
+            widen<T>(raw, qv[j]);
+        } else {
+#pragma unroll
+            for (int e = 0; e < V; ++e) qv[j][e] = 0.f;
+        }
+    }
+    unsigned long long l[kListK];
+#pragma unroll
+    for (int j = 0; j < kListK; ++j) l[j] = 0ull;
+    const int64_t gwarp = static_cast<int64_t>(blockIdx.x) * kWarps + warp;
+    const int64_t nwarps = static_cast<int64_t>(gridDim.x) * kWarps;
+    for (int64_t r0 = gwarp * RIF; r0 < M; r0 += nwarps * RIF) {
+        uint4 raw[RIF][VPL];
+#pragma unroll
+        for (int r = 0; r < RIF; ++r)
+#pragma unroll
+            for (int j = 0; j < VPL; ++j) {
+                const int v = lane + 32 * j;
+                const int64_t row = r0 + r;
+                raw[r][j] = (v < vecs && row < M)
+                                ? __ldg(reinterpret_cast<const uint4 *>(index + row * dim) + v)
+                                : make_uint4(0, 0, 0, 0);
+            }
+#pragma unroll
+        for (int r = 0; r < RIF; ++r) {
+            float acc = 0.f;
+#pragma unroll
+            for (int j = 0; j < VPL; ++j) {
+                float f[V];
+                widen<T>(raw[r][j], f);
+#pragma unroll
+                for (int e = 0; e < V; ++e) acc = fmaf(f[e], qv[j][e], acc);
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+            const int64_t row = r0 + r;
+            if (row < M && !isnan(acc)) list_insert(l, make_key(acc, row));
+        }
+    }
+    if (lane == 0)
+#pragma unroll
+        for (int j = 0; j < kListK; ++j) lists[warp][j] = l[j];
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        unsigned long long m[kListK];
+#pragma unroll
+        for (int j = 0; j < kListK; ++j) m[j] = lists[0][j];
+        for (int w = 1; w < kWarps; ++w)
+#pragma unroll
+            for (int j = 0; j < kListK; ++j) list_insert(m, lists[w][j]);
+#pragma unroll
+        for (int j = 0; j < kListK; ++j)
+            partial[(static_cast<int64_t>(blockIdx.x) * n_queries + q) * kListK + j] = m[j];
+    }
+}
+
+// Merge the per-CTA lists of one query (one thread per query) into its k best.
+__global__ void finalize_topk_kernel(const unsigned long long *__restrict__ partial, int n_parts,
+                                     int n_queries, int k, int64_t *__restrict__ best_idx,
+                                     float *__restrict__ best_score) {
+    const int q = blockIdx.x * blockDim.x + threadIdx.x;
+    if (q >= n_queries) return;
+    unsigned long long l[kListK];
+#pragma unroll
+    for (int j = 0; j < kListK; ++j) l[j] = 0ull;
+    for (int i = 0; i < n_parts; ++i)
+        for (int j = 0; j < kListK; ++j) {
+            const unsigned long long v = partial[(static_cast<int64_t>(i) * n_queries + q) * kListK + j];
+            if (v <= l[kListK - 1]) break;   // each part's list is sorted: the rest is smaller
+            list_insert(l, v);
+        }
+    for (int j = 0; j < k; ++j) {
+        const unsigned long long key = l[j];
+        const int64_t o = static_cast<int64_t>(q) * k + j;
+        if (key == 0ull) {
+            best_idx[o] = -1;
+            if (best_score) best_score[o] = __uint_as_float(0x7fc00000u);
+        } else {
+            best_idx[o] = static_cast<int64_t>(0xffffffffu - static_cast<uint32_t>(key & 0xffffffffu));
+            if (best_score) best_score[o] = unordered_float(static_cast<uint32_t>(key >> 32));
+        }
+    }
+}
+
 int num_sms() {
     static int sms = 0;
     if (sms == 0) {
@@ -232,6 +351,30 @@ bool use_tc(const RetrieveParams &p) {
     return p.dtype != PRECOG_F32 && p.n_queries >= kTcMinQueries && p.M > 0;
 }
 
+template <typename T, int VPL>
+cudaError_t launch_topk_pass(const RetrieveParams &p, int grid, int q, cudaStream_t stream) {
+    gemv_topk_kernel<T, VPL><<<grid, kThreads, 0, stream>>>(
+        static_cast<const T *>(p.index), p.M, p.dim, static_cast<const T *>(p.queries), p.n_queries, q,
+        static_cast<unsigned long long *>(p.workspace));
+    return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t launch_gemv_topk(const RetrieveParams &p, cudaStream_t stream, int grid,
+                             uint64_t *launches) {
+    const int vpl = (p.dim / Vec<T>::n + 31) / 32;
+    cudaError_t e = cudaSuccess;
+    for (int q = 0; q < p.n_queries && e == cudaSuccess; ++q, ++*launches) {
+        if (vpl <= 1) e = launch_topk_pass<T, 1>(p, grid, q, stream);
+        else if (vpl <= 2) e = launch_topk_pass<T, 2>(p, grid, q, stream);
+        else if (vpl <= 3) e = launch_topk_pass<T, 3>(p, grid, q, stream);
+        else if (vpl <= 4) e = launch_topk_pass<T, 4>(p, grid, q, stream);
+        else if (vpl <= 8) e = launch_topk_pass<T, 8>(p, grid, q, stream);
+        else e = launch_topk_pass<T, 16>(p, grid, q, stream);
+    }
+    return e;
+}
+
 }  // namespace
 
 size_t retrieve_workspace_size(int64_t M, int32_t dim, int32_t n_queries) {
@@ -262,6 +405,42 @@ cudaError_t launch_retrieve(const RetrieveParams &p, cudaStream_t stream) {
     if (e == cudaSuccess) {
         finalize_kernel<<<(p.n_queries + 127) / 128, 128, 0, stream>>>(
             static_cast<const unsigned long long *>(p.workspace), parts, p.n_queries, p.best_idx,
+            p.best_score);
+        e = cudaGetLastError();
+        if (e == cudaSuccess) ++launches;
+    }
+    count_launches(launches);
+    return e;
+}
+
+size_t retrieve_topk_workspace_size(int64_t M, int32_t dim, int32_t n_queries) {
+    (void)dim;
+    if (n_queries <= 0) return 0;
+    const int parts = std::max(gemv_grid(M), retrieve_tc_grid(M, num_sms()));
+    return static_cast<size_t>(parts) * n_queries * kListK * sizeof(unsigned long long);
+}
+
+cudaError_t launch_retrieve_topk(const RetrieveParams &p, int k, cudaStream_t stream) {
+    if (p.n_queries == 0) return cudaSuccess;
+    const int sz = p.dtype == PRECOG_F32 ? 4 : 2;
+    if (p.dim * sz / 16 > kMaxVecsPerRow || k < 1 || k > kListK) return cudaErrorInvalidValue;
+    uint64_t launches = 0;
+    cudaError_t e;
+    int parts;
+    if (use_tc(p)) {
+        parts = retrieve_tc_grid(p.M, num_sms());
+        e = launch_retrieve_tc_topk(p, parts, stream, &launches);
+    } else {
+        parts = gemv_grid(p.M);
+        switch (p.dtype) {
+            case PRECOG_F16: e = launch_gemv_topk<__half>(p, stream, parts, &launches); break;
+            case PRECOG_BF16: e = launch_gemv_topk<__nv_bfloat16>(p, stream, parts, &launches); break;
+            default: e = launch_gemv_topk<float>(p, stream, parts, &launches); break;
+        }
+    }
+    if (e == cudaSuccess) {
+        finalize_topk_kernel<<<(p.n_queries + 127) / 128, 128, 0, stream>>>(
+            static_cast<const unsigned long long *>(p.workspace), parts, p.n_queries, k, p.best_idx,
             p.best_score);
         e = cudaGetLastError();
         if (e == cudaSuccess) ++launches;

@@ -77,6 +77,9 @@ __device__ __forceinline__ uint32_t ordered_bits_tc(float s) {
     const uint32_t u = __float_as_uint(s + 0.0f);
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
+__device__ __forceinline__ float unordered_tc(uint32_t k) {
+    return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+}
 
 __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, Smem &sm) {
     for (uint32_t i = 0; i < kWaitLimit; ++i) {
@@ -88,7 +91,25 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, Sm
     return false;
 }
 
-// partial[blockIdx.x * n_queries + q0 + q] = packed best key of this CTA for query q.
+// Sorted insertion into a descending list of packed keys (the smallest drops out).
+template <int K>
+__device__ __forceinline__ void tc_list_insert(unsigned long long (&l)[K], unsigned long long v) {
+#pragma unroll
+    for (int j = K - 1; j > 0; --j) {
+        const bool shift = v > l[j - 1];
+        l[j] = shift ? l[j - 1] : (v > l[j] ? v : l[j]);
+    }
+    l[0] = v > l[0] ? v : l[0];
+}
+
+__device__ __forceinline__ unsigned long long tc_key(float s, int64_t row) {
+    return (static_cast<unsigned long long>(ordered_bits_tc(s)) << 32) |
+           static_cast<unsigned long long>(0xffffffffu - static_cast<uint32_t>(row));
+}
+
+// LIST = 1: partial[blockIdx.x * n_queries + q0 + q] = packed best key of this CTA.
+// LIST > 1: partial[(blockIdx.x * n_queries + q0 + q) * LIST + j] = its LIST best, sorted.
+template <int LIST>
 __global__ void __launch_bounds__(kThreads, 1)
     retrieve_tc_kernel(const __grid_constant__ CUtensorMap tmap_q,
                        const __grid_constant__ CUtensorMap tmap_k, int64_t M, int dim,
@@ -189,6 +210,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int qrow = quarter * 32 + lane;         // query row inside a half
         float best[2] = {-__int_as_float(0x7f800000), -__int_as_float(0x7f800000)};
         int64_t best_row[2] = {-1, -1};
+        unsigned long long lst[2][LIST > 1 ? LIST : 1];
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int j = 0; j < (LIST > 1 ? LIST : 1); ++j) lst[h][j] = 0ull;
         int it = 0;
         for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
             const int acc = it & 1;
@@ -207,19 +233,30 @@ __global__ void __launch_bounds__(kThreads, 1)
                                   static_cast<uint32_t>(acc * 2 * kBN + h * kBN + c0),
                               v);
                     const int64_t rbase = row0 + c0;
-                    if (rbase + 32 <= M) {
+                    if constexpr (LIST == 1) {
+                        if (rbase + 32 <= M) {
 #pragma unroll
-                        for (int j = 0; j < 32; ++j)
-                            if (v[j] > best[h]) {
-                                best[h] = v[j];
-                                best_row[h] = rbase + j;
-                            }
+                            for (int j = 0; j < 32; ++j)
+                                if (v[j] > best[h]) {
+                                    best[h] = v[j];
+                                    best_row[h] = rbase + j;
+                                }
+                        } else {
+#pragma unroll
+                            for (int j = 0; j < 32; ++j)
+                                if (rbase + j < M && v[j] > best[h]) {
+                                    best[h] = v[j];
+                                    best_row[h] = rbase + j;
+                                }
+                        }
                     } else {
+                        // best[h] tracks the list's last score: one compare per column
 #pragma unroll
                         for (int j = 0; j < 32; ++j)
                             if (rbase + j < M && v[j] > best[h]) {
-                                best[h] = v[j];
-                                best_row[h] = rbase + j;
+                                tc_list_insert<LIST>(lst[h], tc_key(v[j], rbase + j));
+                                if (lst[h][LIST - 1] != 0ull)
+                                    best[h] = unordered_tc(static_cast<uint32_t>(lst[h][LIST - 1] >> 32));
                             }
                     }
                 }
@@ -230,7 +267,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         for (int h = 0; h < nhalf; ++h) {
             const int q = h * kBM + qrow;
-            if (q < nq) {
+            if (LIST > 1 && q < nq) {
+#pragma unroll
+                for (int j = 0; j < (LIST > 1 ? LIST : 1); ++j)
+                    partial[(static_cast<int64_t>(blockIdx.x) * n_queries + q0 + q) * LIST + j] = lst[h][j];
+            }
+            if (LIST == 1 && q < nq) {
                 unsigned long long key = 0ull;
                 if (best_row[h] >= 0)
                     key = (static_cast<unsigned long long>(ordered_bits_tc(best[h])) << 32) |
@@ -287,9 +329,9 @@ int retrieve_tc_grid(int64_t M, int sms) {
     return static_cast<int>(ntiles < 1 ? 1 : (ntiles < sms ? ntiles : sms));
 }
 
-// One pass per 256 queries; partial is [grid][n_queries] packed keys.
-cudaError_t launch_retrieve_tc(const RetrieveParams &p, int grid, cudaStream_t stream,
-                               uint64_t *launches) {
+// One pass per 256 queries; partial holds LIST packed keys per (CTA, query).
+template <int LIST>
+cudaError_t launch_tc(const RetrieveParams &p, int grid, cudaStream_t stream, uint64_t *launches) {
     const bool bf16 = p.dtype == PRECOG_BF16;
     CUtensorMap tq, tk;
     if (!make_map(&tq, p.queries, p.n_queries, p.dim, bf16, kBM) ||
@@ -297,11 +339,11 @@ cudaError_t launch_retrieve_tc(const RetrieveParams &p, int grid, cudaStream_t s
         return cudaErrorInvalidValue;
     static int smem_set = 0;
     const int smem = static_cast<int>(retrieve_tc_smem_bytes());
-    cudaError_t e = ensure_smem(reinterpret_cast<const void *>(retrieve_tc_kernel), &smem_set, smem);
+    cudaError_t e = ensure_smem(reinterpret_cast<const void *>(retrieve_tc_kernel<LIST>), &smem_set, smem);
     if (e != cudaSuccess) return e;
     for (int q0 = 0; q0 < p.n_queries; q0 += 2 * kBM) {
         const int nq = p.n_queries - q0 < 2 * kBM ? p.n_queries - q0 : 2 * kBM;
-        retrieve_tc_kernel<<<grid, kThreads, smem, stream>>>(
+        retrieve_tc_kernel<LIST><<<grid, kThreads, smem, stream>>>(
             tq, tk, p.M, p.dim, p.n_queries, q0, nq, bf16,
             static_cast<unsigned long long *>(p.workspace));
         e = cudaGetLastError();
@@ -309,6 +351,16 @@ cudaError_t launch_retrieve_tc(const RetrieveParams &p, int grid, cudaStream_t s
         ++*launches;
     }
     return cudaSuccess;
+}
+
+cudaError_t launch_retrieve_tc(const RetrieveParams &p, int grid, cudaStream_t stream,
+                               uint64_t *launches) {
+    return launch_tc<1>(p, grid, stream, launches);
+}
+
+cudaError_t launch_retrieve_tc_topk(const RetrieveParams &p, int grid, cudaStream_t stream,
+                                    uint64_t *launches) {
+    return launch_tc<8>(p, grid, stream, launches);
 }
 
 cudaError_t retrieve_tc_status_word_read_clear(uint32_t *bits) {

@@ -63,6 +63,7 @@ constexpr int kN = 16;          // state size (N) supported by the kernels
 constexpr int kMaxSlice = 256;  // channels per CTA at most
 constexpr int kBarBytes = 128;  // barrier area at the start of shared memory
 constexpr float kLog2e = 1.4426950408889634f;
+constexpr int kMaxTopk = 8;     // states composed at most by one injection
 
 __device__ __forceinline__ int64_t min64(int64_t a, int64_t b) { return a < b ? a : b; }
 
@@ -536,10 +537,12 @@ __global__ void __launch_bounds__(kMaxSlice / C::CPT, C::MINB)
     bool h0_valid = false;
     int64_t h0_row = 0;
     if constexpr (C::HAS_H0) {
-        h0_row = p.idx ? p.idx[chunk] : chunk;
-        h0_valid = h0_row >= 0 && h0_row < p.bank_entries;
-        if (!h0_valid && !(p.idx && h0_row == -1) && tid == 0)
-            atomicOr(&g_scan_status, PRECOG_DEV_BAD_INDEX);
+        if (p.topk <= 1) {
+            h0_row = p.idx ? p.idx[chunk] : chunk;
+            h0_valid = h0_row >= 0 && h0_row < p.bank_entries;
+            if (!h0_valid && !(p.idx && h0_row == -1) && tid == 0)
+                atomicOr(&g_scan_status, PRECOG_DEV_BAD_INDEX);
+        }
     }
 #pragma unroll
     for (int j = 0; j < CPT; ++j) {
@@ -550,6 +553,52 @@ __global__ void __launch_bounds__(kMaxSlice / C::CPT, C::MINB)
         } else {
 #pragma unroll
             for (int i = 0; i < 8; ++i) h[j][i] = 0;
+        }
+    }
+    if constexpr (C::HAS_H0) {
+        if (p.topk > 1) {
+            // Top-k composition (Sec. 4.4, Eq. smc-fusion): h_init = sum_j w_j bank[row_j],
+            // w = softmax(score / temperature) over the valid rows (row -1 or a NaN score:
+            // weight 0; a row outside the bank: weight 0 and PRECOG_DEV_BAD_INDEX).
+            const int64_t *rows = p.idx + chunk * p.topk;
+            const float *sc = p.topk_scores + chunk * p.topk;
+            float w[kMaxTopk];
+            float smax = -__int_as_float(0x7f800000);
+#pragma unroll
+            for (int k = 0; k < kMaxTopk; ++k) {
+                w[k] = -__int_as_float(0x7f800000);
+                if (k < p.topk) {
+                    const int64_t r = rows[k];
+                    const bool in_bank = r >= 0 && r < p.bank_entries;
+                    if (!in_bank && r != -1 && tid == 0) atomicOr(&g_scan_status, PRECOG_DEV_BAD_INDEX);
+                    const float z = sc[k] * p.inv_temp;
+                    if (in_bank && !isnan(z)) {
+                        w[k] = z;
+                        smax = fmaxf(smax, z);
+                    }
+                }
+            }
+            float wsum = 0.f;
+#pragma unroll
+            for (int k = 0; k < kMaxTopk; ++k) {
+                w[k] = (w[k] == -__int_as_float(0x7f800000)) ? 0.f : ex2((w[k] - smax) * kLog2e);
+                wsum += w[k];
+            }
+#pragma unroll
+            for (int k = 0; k < kMaxTopk; ++k) {
+                if (k >= p.topk || w[k] == 0.f) continue;
+                const float wk = w[k] / wsum;
+                const f2 ww = pack2(wk, wk);
+#pragma unroll
+                for (int j = 0; j < CPT; ++j) {
+                    f2 hk[8];
+                    const int64_t off = ((rows[k] * p.L_bank + p.layer0 + layer) * static_cast<int64_t>(D) +
+                                         d0 + dl + j) * kN;
+                    load_state16(p.bank, p.bank_dtype, off, hk);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) h[j][i] = fma2(ww, hk[i], h[j][i]);
+                }
+            }
         }
     }
     const unsigned wmask = __activemask();
