@@ -17,6 +17,7 @@ module compiles it with gcc and marshals numpy arrays into it.
   lower row), the top-k of Sec. 4.2 / Sec. 5.4.
 * :func:`compose` -- the softmax-weighted state composition of Sec. 4.4
   (multi-chunk extension) and Eq. smc-fusion.
+* :func:`trajectory` -- the K-dial trajectory of Sec. 5.2 (every k-th state).
 """
 from __future__ import annotations
 
@@ -62,6 +63,9 @@ def _load():
         lib.oracle_scan.restype = ctypes.c_int
         lib.oracle_scan.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, p_i64,
                                     p_f64, p_f64, p_f64, p_f64, p_f64, p_f64, p_f64, p_f64]
+        lib.oracle_trajectory.restype = ctypes.c_int
+        lib.oracle_trajectory.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, p_i64,
+                                          p_f64, p_f64, p_f64, p_f64, ctypes.c_int64, p_i64, p_f64]
         lib.oracle_scores.restype = ctypes.c_int
         lib.oracle_scores.argtypes = [ctypes.c_int64, ctypes.c_int64, p_f64, ctypes.c_int64, p_f64,
                                       p_f64]
@@ -199,4 +203,31 @@ def compose(bank_rows, row_scores, temperature=1.0):
     for j in range(len(w)):
         out = out + w[j] * rows[j]
     return out
+
+
+def trajectory_offsets(offsets, stride):
+    """Prefix sums of K_c = ceil(len_c / stride) (entries kept per chunk)."""
+    offsets = np.asarray(offsets, dtype=np.int64)
+    lens = np.diff(offsets)
+    k = (lens + stride - 1) // stride
+    out = np.zeros(len(offsets), dtype=np.int64)
+    np.cumsum(k, out=out[1:])
+    return out
+
+
+def trajectory(x, dt, A, B, offsets, stride):
+    """States after every stride-th token of each chunk and after its last token
+    (Sec. 5.2). Returns ``(traj [entries, D, N], entry_offsets [n_chunks + 1])``."""
+    lib = _load()
+    x, dt, A, B = _f64(x), _f64(dt), _f64(A), _f64(B)
+    offsets = np.ascontiguousarray(np.asarray(offsets, dtype=np.int64))
+    D, N = A.shape
+    eo = trajectory_offsets(offsets, stride)
+    traj = np.zeros((int(eo[-1]), D, N), dtype=np.float64)
+    p64, pi = ctypes.c_double, ctypes.c_int64
+    rc = lib.oracle_trajectory(D, N, len(offsets) - 1, _ptr(offsets, pi), _ptr(x, p64), _ptr(dt, p64),
+                               _ptr(A, p64), _ptr(B, p64), stride, _ptr(eo, pi), _ptr(traj, p64))
+    if rc != 0:
+        raise ValueError(f"oracle_trajectory rejected its arguments (rc={rc})")
+    return traj, eo
 

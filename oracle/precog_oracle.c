@@ -149,3 +149,55 @@ int oracle_scores(int64_t M, int64_t dim, const double *index, int64_t Q,
     return ORACLE_OK;
 }
 
+/*
+ * oracle_trajectory: the K-dial trajectory of Sec. 5.2 (Eq. smc-trajectory):
+ * roll each chunk from the zero state as oracle_scan does and keep the state
+ * after every stride-th token, plus the final state when the chunk length is
+ * not a multiple of stride. Chunk c keeps K_c = ceil(len_c / stride) states
+ * (K = N_c / k in the paper's notation; stride >= len_c keeps only the final
+ * state, the per-chunk PRECOG state).
+ *   entry_offsets [n_chunks+1]  prefix sums of K_c
+ *   traj_out      [entry_offsets[n_chunks]][D][N]; entry entry_offsets[c] + j
+ *                 is the state after token min((j+1)*stride, len_c) of chunk c
+ */
+int oracle_trajectory(int64_t D, int64_t N, int64_t n_chunks, const int64_t *offsets,
+                      const double *x, const double *dt, const double *A, const double *B,
+                      int64_t stride, const int64_t *entry_offsets, double *traj_out)
+{
+    if (D <= 0 || N <= 0 || n_chunks < 0 || stride < 1 || offsets == NULL ||
+        entry_offsets == NULL || traj_out == NULL)
+        return ORACLE_BAD_ARG;
+    for (int64_t c = 0; c < n_chunks; ++c) {
+        const int64_t len = offsets[c + 1] - offsets[c];
+        if (len < 0 || entry_offsets[c + 1] - entry_offsets[c] != (len + stride - 1) / stride)
+            return ORACLE_BAD_ARG;
+    }
+    if (N > 64)
+        return ORACLE_BAD_ARG;
+    for (int64_t c = 0; c < n_chunks; ++c) {
+        for (int64_t d = 0; d < D; ++d) {
+            double h[64];
+            for (int64_t n = 0; n < N; ++n)
+                h[n] = 0.0;
+            int64_t j = 0;
+            for (int64_t t = offsets[c]; t < offsets[c + 1]; ++t) {
+                const double dt_td = dt[t * D + d];
+                const double x_td = x[t * D + d];
+                for (int64_t n = 0; n < N; ++n) {
+                    const double alpha = exp(dt_td * A[d * N + n]);
+                    const double beta = B[t * N + n] * x_td * dt_td;
+                    h[n] = h[n] * alpha + beta;
+                }
+                const int64_t step = t - offsets[c] + 1;
+                if (step % stride == 0 || t + 1 == offsets[c + 1]) {
+                    double *e = traj_out + ((entry_offsets[c] + j) * D + d) * N;
+                    for (int64_t n = 0; n < N; ++n)
+                        e[n] = h[n];
+                    ++j;
+                }
+            }
+        }
+    }
+    return ORACLE_OK;
+}
+

@@ -358,3 +358,29 @@ def test_composition_commutes_with_the_scan():
     parts = [oracle.rollout(x, dt, A, B, C, h0=hs[j], want_y=True) for j in range(3)]
     np.testing.assert_allclose(h_comp, sum(w[j] * parts[j][0] for j in range(3)), rtol=1e-11, atol=1e-12)
     np.testing.assert_allclose(y_comp, sum(w[j] * parts[j][1] for j in range(3)), rtol=1e-11, atol=1e-12)
+
+
+# ---------------------------------------------------------------- K-dial trajectory
+
+
+@pytest.mark.parametrize("stride", [1, 3, 7, 50])
+def test_trajectory_is_prefix_rollouts(stride):
+    """Entry j of chunk c is S(0, c_{1:t}) with t = min((j+1) * stride, len_c): brute
+    force by rolling every prefix separately; the last entry is the chunk's final state
+    (K = 1 is the PRECOG state, Sec. 5.2); empty chunks keep nothing."""
+    D, N = 3, 4
+    lens = [10, 0, 1, 21, 7]
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    x, dt, A, B, _ = _rand_inputs(int(off[-1]), D, N, seed=stride)
+    traj, eo = oracle.trajectory(x, dt, A, B, off, stride)
+    finals, _ = oracle.scan(x, dt, A, B, off)
+    for c, L in enumerate(lens):
+        K = -(-L // stride)
+        assert eo[c + 1] - eo[c] == K
+        for j in range(K):
+            t = min((j + 1) * stride, L)
+            s = off[c]
+            ref, _ = oracle.rollout(x[s:s + t], dt[s:s + t], A, B[s:s + t])
+            np.testing.assert_allclose(traj[eo[c] + j], ref, rtol=1e-12, atol=1e-14)
+        if K:
+            np.testing.assert_array_equal(traj[eo[c + 1] - 1], finals[c])
