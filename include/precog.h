@@ -133,6 +133,28 @@ precog_status precog_encode_chunks(const precog_scan_inputs *in, const int64_t *
                                    void *y_out, int32_t y_dtype, void *stream);
 
 /*
+ * precog_encode_trajectory -- the K-dial state trajectory of SMC (Sec. 5.2,
+ * Eq. smc-trajectory): scan every chunk from the zero state like
+ * precog_encode_chunks and keep the state after every `stride`-th token and
+ * after the chunk's last token. Chunk c keeps K_c = ceil(len_c / stride)
+ * states (K = N_c / k in the paper; stride 1 keeps every state, stride >=
+ * len_c keeps only the final, PRECOG state). Uses the direct update.
+ *   d_entry_offsets  device int64 [n_chunks+1]: prefix sums of K_c; a chunk
+ *                    whose count disagrees with its length is skipped and
+ *                    flags PRECOG_DEV_BAD_OFFSETS
+ *   traj_out         device [d_entry_offsets[n_chunks]][L_total][D][N] in
+ *                    traj_dtype (F32 or BF16); entry d_entry_offsets[c] + j is
+ *                    the state after token min((j+1)*stride, len_c) of chunk c,
+ *                    written for layers layer0 .. layer0+L-1
+ * Other arguments as precog_encode_chunks.
+ */
+precog_status precog_encode_trajectory(const precog_scan_inputs *in, const int64_t *d_offsets,
+                                       int64_t n_chunks, int64_t T_tot, int64_t stride,
+                                       const int64_t *d_entry_offsets, void *traj_out,
+                                       int32_t traj_dtype, int32_t layer0, int32_t L_total,
+                                       void *stream);
+
+/*
  * precog_retrieve -- query-time retrieval (Sec. 4.2): for every query q the
  * row i* of the key index with the highest dot product <query_q, key_i>
  * (unit-norm keys and queries make this the cosine similarity of the paper).

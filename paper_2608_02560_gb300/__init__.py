@@ -9,6 +9,7 @@ loudly: there is no CPU fallback.
 Functions carry the C names:
 
 * :func:`precog_encode_chunks`    -- offline indexing (Sec. 4.2)
+* :func:`precog_encode_trajectory` -- K-dial trajectory capture (Sec. 5.2)
 * :func:`precog_retrieve`         -- exact top-1 retrieval (Sec. 4.2)
 * :func:`precog_prefill_from_state` -- injection (Eq. 2) + query prefill
 * :func:`precog_retrieve_topk`    -- top-k retrieval (Sec. 4.2 / 5.4)
@@ -70,6 +71,9 @@ def load_library(path: str = LIB_PATH):
     lib.precog_prefill_from_state.restype = i32
     lib.precog_prefill_from_state.argtypes = [ctypes.POINTER(ScanInputs), i32, i32, vp, i32, i64,
                                               i32, i32, vp, vp, i32, vp, i32, vp]
+    lib.precog_encode_trajectory.restype = i32
+    lib.precog_encode_trajectory.argtypes = [ctypes.POINTER(ScanInputs), vp, i64, i64, i64, vp, vp,
+                                             i32, i32, i32, vp]
     lib.precog_retrieve_topk.restype = i32
     lib.precog_retrieve_topk.argtypes = [vp, i32, i64, i32, vp, i32, i32, vp, vp, vp, sz, vp]
     lib.precog_retrieve_topk_workspace_size.restype = sz
@@ -166,6 +170,18 @@ def precog_encode_chunks(inputs: ScanInputs, offsets, T_tot: int, states_out=Non
         ctypes.byref(inputs), _ptr(offsets), n_chunks, T_tot, _ptr(states_out),
         _dtype_code(states_out) if states_out is not None else PRECOG_F32, layer0, L_total,
         _ptr(y_out), _dtype_code(y_out) if y_out is not None else PRECOG_F32, _stream(stream)))
+
+
+def precog_encode_trajectory(inputs: ScanInputs, offsets, T_tot: int, stride: int, entry_offsets,
+                             traj_out, layer0: int = 0, L_total: int | None = None, stream=None):
+    """Keep the state after every ``stride``-th token and the last token of each chunk in
+    ``traj_out [entries, L_total, D, N]`` (K-dial trajectory, Sec. 5.2)."""
+    lib = load_library()
+    if L_total is None:
+        L_total = inputs.n_layers
+    _check(lib.precog_encode_trajectory(
+        ctypes.byref(inputs), _ptr(offsets), offsets.numel() - 1, T_tot, stride, _ptr(entry_offsets),
+        _ptr(traj_out), _dtype_code(traj_out), layer0, L_total, _stream(stream)))
 
 
 def precog_retrieve_workspace_size(M: int, dim: int, n_queries: int) -> int:

@@ -196,6 +196,37 @@ precog_status precog_prefill_from_state(const precog_scan_inputs *in, int32_t n_
     return ok();
 }
 
+precog_status precog_encode_trajectory(const precog_scan_inputs *in, const int64_t *d_offsets,
+                                       int64_t n_chunks, int64_t T_tot, int64_t stride,
+                                       const int64_t *d_entry_offsets, void *traj_out,
+                                       int32_t traj_dtype, int32_t layer0, int32_t L_total,
+                                       void *stream) {
+    if (T_tot < 0) return fail(PRECOG_ERR_INVALID_ARG, "T_tot must be >= 0");
+    precog_status s = check_scan_inputs(in, T_tot, false);
+    if (s != PRECOG_OK) return s;
+    if (n_chunks < 0) return fail(PRECOG_ERR_INVALID_ARG, "n_chunks must be >= 0");
+    if (stride < 1) return fail(PRECOG_ERR_INVALID_ARG, "stride must be >= 1");
+    if (d_offsets == nullptr || d_entry_offsets == nullptr)
+        return fail(PRECOG_ERR_INVALID_ARG, "d_offsets and d_entry_offsets must be non-NULL");
+    if (traj_out == nullptr || !state_dtype_ok(traj_dtype) || !aligned16(traj_out))
+        return fail(PRECOG_ERR_INVALID_ARG, "traj_out must be a 16-byte aligned F32 or BF16 array");
+    if (layer0 < 0 || L_total < 1 || layer0 + in->n_layers > L_total)
+        return fail(PRECOG_ERR_INVALID_ARG, "layers [layer0, layer0+n_layers) exceed L_total");
+    if (n_chunks == 0) return ok();
+    precog::ScanParams p = base_params(in, T_tot);
+    p.offsets = d_offsets;
+    p.n_chunks = n_chunks;
+    p.L_out = L_total;
+    p.layer0 = layer0;
+    p.traj = traj_out;
+    p.traj_dtype = traj_dtype;
+    p.traj_stride = stride;
+    p.traj_offsets = d_entry_offsets;
+    cudaError_t e = precog::launch_scan(p, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "trajectory launch");
+    return ok();
+}
+
 precog_status precog_prefill_composed(const precog_scan_inputs *in, int32_t n_queries, int32_t T_q,
                                      const void *bank, int32_t bank_dtype, int64_t bank_entries,
                                      int32_t L_bank, int32_t layer0, int32_t k,

@@ -40,6 +40,11 @@ struct ScanParams {
     int32_t layer0;           // first layer of the bank / output entries
     void *y;                  // [L][T_tot][D] or nullptr
     int32_t y_dtype;
+    // trajectory (K-dial): states after every traj_stride-th token and the last
+    void *traj;               // [entries][L_out][D][N] or nullptr
+    int32_t traj_dtype;
+    int64_t traj_stride;
+    const int64_t *traj_offsets;  // [n_chunks+1] first entry of each chunk
 };
 
 // Kernel launches made by this library since the process started.

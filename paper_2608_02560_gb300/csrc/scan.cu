@@ -71,14 +71,21 @@ enum Mode { kGeneral = 0, kPower = 1 };
 
 // Compile-time shape of one kernel instantiation.
 template <typename TIn_, bool HAS_Y_, bool HAS_H0_, int MODE_, int CPT_, int TILE_, int STAGES_,
-          int MINB_>
+          int MINB_, bool TRAJ_ = false>
 struct Cfg {
     using TIn = TIn_;
     static constexpr bool HAS_Y = HAS_Y_, HAS_H0 = HAS_H0_;
+    static constexpr bool TRAJ = TRAJ_;     // keep every stride-th state (K-dial, Sec. 5.2)
     static constexpr int MODE = MODE_, CPT = CPT_, TILE = TILE_, STAGES = STAGES_, MINB = MINB_;
     static constexpr bool CONV = !std::is_same<TIn_, float>::value;
     static constexpr int SZ = sizeof(TIn_);
-    static constexpr bool RESCALED = MODE_ == kPower && !HAS_Y_;
+    static constexpr bool RESCALED = MODE_ == kPower && !HAS_Y_ && !TRAJ_;
+};
+
+// Where the next trajectory state goes: entry index and tokens left until it.
+struct TrajCursor {
+    int64_t entry;
+    int64_t left;
 };
 
 struct StageLayout {
@@ -226,7 +233,9 @@ __device__ __forceinline__ void scan_tile_direct(const unsigned char *st, const 
                                                  int DS, int dl, int ntok,
                                                  f2 (&h)[C::CPT][8], const float (&kpow)[C::CPT],
                                                  const f2 (&kgen)[C::CPT][8], void *yrow,
-                                                 int y_dtype, int64_t y_stride) {
+                                                 int y_dtype, int64_t y_stride,
+                                                 const ScanParams &p, TrajCursor &tc,
+                                                 int64_t tok_left, int traj_layer, int dglob) {
     constexpr int CPT = C::CPT;
     const float *bsrc = reinterpret_cast<const float *>(st + (C::CONV ? lay.bf : lay.bs));
     const float *csrc = reinterpret_cast<const float *>(st + (C::CONV ? lay.cf : lay.cs));
@@ -287,6 +296,19 @@ __device__ __forceinline__ void scan_tile_direct(const unsigned char *st, const 
                     *reinterpret_cast<uint2 *>(dst) = make_uint2(
                         *reinterpret_cast<uint32_t *>(&p0), *reinterpret_cast<uint32_t *>(&p1));
                 }
+            }
+        }
+        if constexpr (C::TRAJ) {
+            // after every stride-th token and after the chunk's last token (uniform)
+            if (--tc.left == 0 || t + 1 == tok_left) {
+#pragma unroll
+                for (int j = 0; j < CPT; ++j)
+                    store_state16(p.traj, p.traj_dtype,
+                                  ((tc.entry * p.L_out + traj_layer) * static_cast<int64_t>(p.D) + dglob + j) *
+                                      kN,
+                                  h[j]);
+                ++tc.entry;
+                tc.left = p.traj_stride;
             }
         }
     }
@@ -464,6 +486,17 @@ __global__ void __launch_bounds__(kMaxSlice / C::CPT, C::MINB)
             return;
         }
         len = end - start;
+    }
+    TrajCursor tcur{0, 0};
+    if constexpr (C::TRAJ) {
+        // chunk c keeps ceil(len / stride) states starting at entry traj_offsets[c]
+        const int64_t e0 = p.traj_offsets[chunk], e1 = p.traj_offsets[chunk + 1];
+        if (e1 - e0 != (len + p.traj_stride - 1) / p.traj_stride) {
+            if (tid == 0) atomicOr(&g_scan_status, PRECOG_DEV_BAD_OFFSETS);
+            return;
+        }
+        tcur.entry = e0;
+        tcur.left = p.traj_stride;
     }
     const int d0 = slice * DS;
     const int dl = tid * CPT;
@@ -645,7 +678,8 @@ __global__ void __launch_bounds__(kMaxSlice / C::CPT, C::MINB)
         if constexpr (C::RESCALED) {
             scan_tile_rescaled<C>(st, lay, DS, dl, ntok, h, Lw, kk, wmask);
         } else {
-            scan_tile_direct<C>(st, lay, DS, dl, ntok, h, kpow, kgen, yrow, p.y_dtype, y_stride);
+            scan_tile_direct<C>(st, lay, DS, dl, ntok, h, kpow, kgen, yrow, p.y_dtype, y_stride, p, tcur,
+                                len - k * TILE, p.layer0 + layer, d0 + dl);
         }
         if (C::HAS_Y) {
             yrow = (p.y_dtype == PRECOG_F32)
@@ -703,9 +737,16 @@ cudaError_t launch_cfg(const ScanParams &p, cudaStream_t stream) {
 
 // Shapes: the rescaled capture kernel (the corpus-encode hot loop) and the
 // direct kernels (readout, prefill, general A).
-template <typename TIn, bool HAS_Y, bool HAS_H0, int MODE>
+template <typename TIn, bool HAS_Y, bool HAS_H0, int MODE, bool TRAJ = false>
 cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
-    if constexpr (MODE == kPower && !HAS_Y) {
+    if constexpr (TRAJ) {
+        // trajectory capture uses the direct update (the state is needed every stride tokens)
+        if constexpr (MODE == kPower)
+            return launch_cfg<Cfg<TIn, false, false, MODE, PRECOG_DIRECT_CPT, PRECOG_DIRECT_TILE,
+                                  PRECOG_DIRECT_STAGES, PRECOG_DIRECT_MINB, true>>(p, stream);
+        else
+            return launch_cfg<Cfg<TIn, false, false, MODE, 2, 16, 4, 3, true>>(p, stream);
+    } else if constexpr (MODE == kPower && !HAS_Y) {
         return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
                               PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB>>(p, stream);
     } else {
@@ -721,6 +762,7 @@ cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
 
 template <typename TIn, int MODE>
 cudaError_t launch_mode(const ScanParams &p, cudaStream_t stream) {
+    if (p.traj != nullptr) return launch_t<TIn, false, false, MODE, true>(p, stream);
     const bool has_y = p.y != nullptr;
     const bool has_h0 = p.bank != nullptr;
     if (has_y)
