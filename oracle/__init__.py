@@ -18,6 +18,9 @@ module compiles it with gcc and marshals numpy arrays into it.
 * :func:`compose` -- the softmax-weighted state composition of Sec. 4.4
   (multi-chunk extension) and Eq. smc-fusion.
 * :func:`trajectory` -- the K-dial trajectory of Sec. 5.2 (every k-th state).
+* :func:`smc_route` -- two-level cluster routing of Sec. 5.1 (Eqs. smc-domain,
+  smc-sub).
+* :func:`smc_consolidate` -- the semantic-state EMA of Sec. 5.3 (Eq. smc-ema).
 """
 from __future__ import annotations
 
@@ -230,4 +233,37 @@ def trajectory(x, dt, A, B, offsets, stride):
     if rc != 0:
         raise ValueError(f"oracle_trajectory rejected its arguments (rc={rc})")
     return traj, eo
+
+
+def smc_route(embeddings, domain_protos, sub_protos, J):
+    """m* = argmax_m <e, p_m>, then j* = argmax_{j < J[m*]} <e, q_{m*, j}> (Sec. 5.1);
+    both argmaxes keep the lowest index on ties and never pick a NaN score.
+    ``sub_protos [M, J_max, dim]``. Returns ``(m* int64 [n], j* int64 [n])``; -1 when no
+    comparable score exists."""
+    emb = _f64(embeddings)
+    if emb.ndim == 1:
+        emb = emb.reshape(1, -1)
+    sub = _f64(sub_protos)
+    m_idx, _ = retrieve(domain_protos, emb)
+    j_idx = np.full(emb.shape[0], -1, dtype=np.int64)
+    for c in range(emb.shape[0]):
+        m = int(m_idx[c])
+        if m < 0 or int(J[m]) <= 0:
+            continue
+        jj, _ = retrieve(sub[m, : int(J[m])], emb[c:c + 1])
+        j_idx[c] = jj[0]
+    return m_idx, j_idx
+
+
+def smc_consolidate(semantic, states, slots, alpha):
+    """For c = 0, 1, ... in order: s[slot_c] <- (1 - alpha) s[slot_c] + alpha h^(c)
+    (Eq. smc-ema); a slot of -1 (a forgetting candidate) deposits nothing. Returns the
+    updated table in double."""
+    out = _f64(semantic).copy()
+    h = _f64(states)
+    for c, slot in enumerate(np.asarray(slots, dtype=np.int64)):
+        if slot < 0:
+            continue
+        out[slot] = (1.0 - alpha) * out[slot] + alpha * h[c]
+    return out
 

@@ -384,3 +384,37 @@ def test_trajectory_is_prefix_rollouts(stride):
             np.testing.assert_allclose(traj[eo[c] + j], ref, rtol=1e-12, atol=1e-14)
         if K:
             np.testing.assert_array_equal(traj[eo[c + 1] - 1], finals[c])
+
+
+# ---------------------------------------------------------------- SMC routing and consolidation
+
+
+def test_smc_route_two_levels():
+    """Hand-built prototypes: the domain is the best prototype, the sub-cluster the best
+    among that domain's J[m] sub-prototypes only (not the global best sub-prototype)."""
+    P = np.array([[1.0, 0.0, 0.0], [0.0, 1.0, 0.0], [0.0, 0.0, 1.0]])
+    Qs = np.zeros((3, 2, 3))
+    Qs[0] = [[1.0, 1.0, 0.0], [1.0, -1.0, 0.0]]
+    Qs[1] = [[0.0, 1.0, 5.0], [0.0, 0.0, 0.0]]          # second entry unused (J[1] = 1)
+    Qs[2] = [[0.0, 0.0, 1.0], [9.0, 9.0, 9.0]]
+    J = [2, 1, 2]
+    e = np.array([[0.9, -0.2, 0.1], [0.1, 0.8, 0.7], [0.2, 0.1, 0.95], [1.0, 1.0, 0.0]])
+    m, j = oracle.smc_route(e, P, Qs, J)
+    assert list(m) == [0, 1, 2, 0]                      # ties (row 3) go to the lower domain
+    assert list(j) == [1, 0, 1, 0]
+
+
+def test_smc_consolidate_closed_form():
+    """Constant deposits h into one slot n times from s0: s_n = (1-a)^n s0 + (1-(1-a)^n) h;
+    a = 1 keeps the last deposit; slot -1 deposits nothing; other slots are untouched."""
+    rng = np.random.default_rng(2)
+    s0 = rng.standard_normal((3, 5))
+    h = rng.standard_normal(5)
+    a, n = 0.3, 7
+    out = oracle.smc_consolidate(s0, np.tile(h, (n + 1, 1)), [1] * n + [-1], a)
+    np.testing.assert_allclose(out[1], (1 - a) ** n * s0[1] + (1 - (1 - a) ** n) * h, rtol=1e-12)
+    np.testing.assert_array_equal(out[[0, 2]], s0[[0, 2]])
+    hs = rng.standard_normal((4, 5))
+    out = oracle.smc_consolidate(s0, hs, [2, 0, 2, 0], 1.0)
+    np.testing.assert_array_equal(out[2], hs[2])
+    np.testing.assert_array_equal(out[0], hs[3])
