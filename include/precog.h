@@ -273,6 +273,43 @@ precog_status precog_prefill_composed(const precog_scan_inputs *in, int32_t n_qu
                                       int32_t state_dtype, void *stream);
 
 /*
+ * precog_smc_route -- two-level cluster routing of Structured Memory
+ * Consolidation (Sec. 5.1, Eqs. smc-domain and smc-sub): for every embedding e
+ * (a chunk's or an opening utterance's text embedding)
+ *   m* = argmax_m <e, p_m>,   j* = argmax_{j < J[m*]} <e, q_{m*, j}>,
+ * dot products accumulated in fp32 with a fixed order; ties go to the lower
+ * index; NaN never wins; -1 when nothing is comparable.
+ *   embeddings   device [n][dim]; domain_protos device [M][dim];
+ *                sub_protos device [M][J_max][dim]; all of `dtype` (F16/BF16/F32)
+ *   d_J          device int32 [M]: sub-clusters in use per domain (<= J_max;
+ *                larger values flag PRECOG_DEV_BAD_INDEX and route to none)
+ *   d_domain, d_sub  device int32 [n] (written)
+ *   d_slot       device int64 [n]: m* * J_max + j*, the row of the semantic-
+ *                state table (or -1); may be NULL
+ */
+precog_status precog_smc_route(const void *embeddings, int32_t dtype, int64_t n, int32_t dim,
+                               const void *domain_protos, int32_t M, const void *sub_protos,
+                               int32_t J_max, const int32_t *d_J, int32_t *d_domain, int32_t *d_sub,
+                               int64_t *d_slot, void *stream);
+
+/*
+ * precog_smc_consolidate -- semantic consolidation (Sec. 5.3, Eq. smc-ema): for
+ * c = 0, 1, ..., n-1 in order, s[slot_c] <- (1 - alpha) s[slot_c] + alpha h_c,
+ * in fp32. A slot of -1 (a forgetting candidate) deposits nothing; a slot
+ * outside [0, n_slots) deposits nothing and flags PRECOG_DEV_BAD_INDEX.
+ *   semantic     device fp32 [n_slots][state_elems], updated in place (e.g. the
+ *                [slots][L][D][N] semantic-state table; inject a row with
+ *                precog_prefill_from_state for O(1) session initialisation)
+ *   states       device [n][state_elems] in states_dtype (F32 or BF16), e.g. the
+ *                chunks' K = 1 states from precog_encode_chunks
+ *   d_slots      device int64 [n], e.g. precog_smc_route's d_slot
+ *   alpha        in (0, 1]
+ */
+precog_status precog_smc_consolidate(float *semantic, int64_t n_slots, int64_t state_elems,
+                                     const void *states, int32_t states_dtype, const int64_t *d_slots,
+                                     int64_t n, float alpha, void *stream);
+
+/*
  * precog_device_status -- synchronise `stream`, then report and clear the
  * device status word shared by all calls on this device. *bits_out receives
  * the PRECOG_DEV_* bits seen since the last clear. Returns PRECOG_OK when no

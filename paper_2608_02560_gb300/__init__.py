@@ -14,6 +14,7 @@ Functions carry the C names:
 * :func:`precog_prefill_from_state` -- injection (Eq. 2) + query prefill
 * :func:`precog_retrieve_topk`    -- top-k retrieval (Sec. 4.2 / 5.4)
 * :func:`precog_prefill_composed` -- softmax-weighted top-k injection (Sec. 4.4) + prefill
+* :func:`precog_smc_route`, :func:`precog_smc_consolidate` -- SMC (Sec. 5)
 * :func:`precog_device_status`    -- device-side status word
 """
 from __future__ import annotations
@@ -74,6 +75,10 @@ def load_library(path: str = LIB_PATH):
     lib.precog_encode_trajectory.restype = i32
     lib.precog_encode_trajectory.argtypes = [ctypes.POINTER(ScanInputs), vp, i64, i64, i64, vp, vp,
                                              i32, i32, i32, vp]
+    lib.precog_smc_route.restype = i32
+    lib.precog_smc_route.argtypes = [vp, i32, i64, i32, vp, i32, vp, i32, vp, vp, vp, vp, vp]
+    lib.precog_smc_consolidate.restype = i32
+    lib.precog_smc_consolidate.argtypes = [vp, i64, i64, vp, i32, vp, i64, ctypes.c_float, vp]
     lib.precog_retrieve_topk.restype = i32
     lib.precog_retrieve_topk.argtypes = [vp, i32, i64, i32, vp, i32, i32, vp, vp, vp, sz, vp]
     lib.precog_retrieve_topk_workspace_size.restype = sz
@@ -242,6 +247,27 @@ def precog_prefill_composed(inputs: ScanInputs, n_queries: int, T_q: int, bank, 
         k, _ptr(idx), _ptr(scores), temperature, _ptr(y_out),
         _dtype_code(y_out) if y_out is not None else PRECOG_F32, _ptr(state_out),
         _dtype_code(state_out) if state_out is not None else PRECOG_F32, _stream(stream)))
+
+
+def precog_smc_route(embeddings, domain_protos, sub_protos, J, out_domain, out_sub, out_slot=None,
+                     stream=None):
+    """Two-level routing (Sec. 5.1): ``sub_protos [M, J_max, dim]``, ``J`` int32 [M]."""
+    lib = load_library()
+    n, dim = embeddings.shape
+    M, J_max = sub_protos.shape[0], sub_protos.shape[1]
+    _check(lib.precog_smc_route(
+        _ptr(embeddings), _dtype_code(embeddings), n, dim, _ptr(domain_protos), M, _ptr(sub_protos),
+        J_max, _ptr(J), _ptr(out_domain), _ptr(out_sub), _ptr(out_slot), _stream(stream)))
+
+
+def precog_smc_consolidate(semantic, states, slots, alpha: float, stream=None):
+    """EMA of deposited states into the fp32 semantic table, in deposit order (Sec. 5.3)."""
+    lib = load_library()
+    n_slots = semantic.shape[0]
+    elems = semantic[0].numel() if n_slots else 0
+    _check(lib.precog_smc_consolidate(
+        _ptr(semantic), n_slots, elems, _ptr(states), _dtype_code(states), _ptr(slots),
+        states.shape[0], alpha, _stream(stream)))
 
 
 def precog_device_status(stream=None):

@@ -366,6 +366,42 @@ precog_status precog_retrieve(const void *index, int32_t index_dtype, int64_t M,
     return ok();
 }
 
+precog_status precog_smc_route(const void *embeddings, int32_t dtype, int64_t n, int32_t dim,
+                               const void *domain_protos, int32_t M, const void *sub_protos,
+                               int32_t J_max, const int32_t *d_J, int32_t *d_domain, int32_t *d_sub,
+                               int64_t *d_slot, void *stream) {
+    if (dtype_size(dtype) == 0) return fail(PRECOG_ERR_UNSUPPORTED, "dtype must be F16, BF16 or F32");
+    if (n < 0 || dim < 1 || M < 0 || J_max < 0)
+        return fail(PRECOG_ERR_INVALID_ARG, "n, M, J_max must be >= 0 and dim >= 1");
+    if (n == 0) return ok();
+    if (n > 0x7fffffffLL * 8) return fail(PRECOG_ERR_UNSUPPORTED, "too many embeddings");
+    if (embeddings == nullptr || d_domain == nullptr || d_sub == nullptr ||
+        (M > 0 && (domain_protos == nullptr || d_J == nullptr)) ||
+        (M > 0 && J_max > 0 && sub_protos == nullptr))
+        return fail(PRECOG_ERR_INVALID_ARG, "a required pointer is NULL");
+    cudaError_t e = precog::launch_smc_route(embeddings, dtype, n, dim, domain_protos, M, sub_protos,
+                                             J_max, d_J, d_domain, d_sub, d_slot,
+                                             static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "smc route launch");
+    return ok();
+}
+
+precog_status precog_smc_consolidate(float *semantic, int64_t n_slots, int64_t state_elems,
+                                     const void *states, int32_t states_dtype, const int64_t *d_slots,
+                                     int64_t n, float alpha, void *stream) {
+    if (!state_dtype_ok(states_dtype)) return fail(PRECOG_ERR_UNSUPPORTED, "states_dtype must be F32 or BF16");
+    if (n_slots < 0 || state_elems < 0 || n < 0)
+        return fail(PRECOG_ERR_INVALID_ARG, "sizes must be >= 0");
+    if (!(alpha > 0.f && alpha <= 1.f)) return fail(PRECOG_ERR_INVALID_ARG, "alpha must be in (0, 1]");
+    if (n == 0 || state_elems == 0) return ok();
+    if (semantic == nullptr || states == nullptr || d_slots == nullptr)
+        return fail(PRECOG_ERR_INVALID_ARG, "semantic, states and d_slots must be non-NULL");
+    cudaError_t e = precog::launch_smc_consolidate(semantic, n_slots, state_elems, states, states_dtype,
+                                                   d_slots, n, alpha, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "smc consolidate launch");
+    return ok();
+}
+
 precog_status precog_device_status(void *stream, uint32_t *bits_out) {
     if (bits_out == nullptr) return fail(PRECOG_ERR_INVALID_ARG, "bits_out is NULL");
     *bits_out = 0;
@@ -376,7 +412,10 @@ precog_status precog_device_status(void *stream, uint32_t *bits_out) {
     if (e != cudaSuccess) return cuda_fail(e, "read scan status");
     e = precog::retrieve_status_word_read_clear(&b);
     if (e != cudaSuccess) return cuda_fail(e, "read retrieve status");
-    *bits_out = a | b;
+    uint32_t c = 0;
+    e = precog::smc_status_word_read_clear(&c);
+    if (e != cudaSuccess) return cuda_fail(e, "read smc status");
+    *bits_out = a | b | c;
     if (*bits_out == 0) return ok();
     if (*bits_out & PRECOG_DEV_TIMEOUT)
         return fail(PRECOG_ERR_TIMEOUT, "a device-side wait gave up (bits 0x%x)", *bits_out);

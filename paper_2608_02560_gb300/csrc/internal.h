@@ -87,4 +87,13 @@ cudaError_t launch_retrieve_tc_topk(const RetrieveParams &p, int grid, cudaStrea
 cudaError_t launch_retrieve(const RetrieveParams &p, cudaStream_t stream);
 cudaError_t retrieve_status_word_read_clear(uint32_t *bits);
 
+// SMC primitives (smc.cu)
+cudaError_t launch_smc_route(const void *emb, int dtype, int64_t n, int dim, const void *dom, int M,
+                             const void *sub, int J_max, const int32_t *J, int32_t *out_m,
+                             int32_t *out_j, int64_t *out_slot, cudaStream_t stream);
+cudaError_t launch_smc_consolidate(float *sem, int64_t n_slots, int64_t elems, const void *states,
+                                   int states_dtype, const int64_t *slots, int64_t n, float alpha,
+                                   cudaStream_t stream);
+cudaError_t smc_status_word_read_clear(uint32_t *bits);
+
 }  // namespace precog

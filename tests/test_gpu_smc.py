@@ -1,0 +1,74 @@
+"""GPU parity of the SMC primitives (Sec. 5): two-level routing, semantic-state EMA and
+O(1) session initialisation by injecting a consolidated state."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from tests._util import TOL_F32, rel_err, to_np
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("dtype_name", ["float32", "float16", "bfloat16"])
+def test_route_exact_integer_scores(cuda_device, dtype_name):
+    """Small-integer embeddings and prototypes (exact scores, frequent ties): domain and
+    sub-cluster must equal the oracle's; J[m] limits the sub-clusters searched."""
+    import torch
+    import paper_2608_02560_gb300 as pg
+    dtype = getattr(torch, dtype_name)
+    rng = np.random.default_rng(7)
+    n, dim, M, J_max = 3000, 384, 5, 4
+    emb = rng.integers(-2, 3, size=(n, dim)).astype(np.float32)
+    P = rng.integers(-2, 3, size=(M, dim)).astype(np.float32)
+    S = rng.integers(-2, 3, size=(M, J_max, dim)).astype(np.float32)
+    J = np.array([4, 1, 3, 0, 2], dtype=np.int32)
+    t = lambda a, dt=dtype: torch.from_numpy(np.ascontiguousarray(a)).to(cuda_device, dt)
+    dm = torch.empty(n, dtype=torch.int32, device=cuda_device)
+    dj = torch.empty(n, dtype=torch.int32, device=cuda_device)
+    slot = torch.empty(n, dtype=torch.int64, device=cuda_device)
+    pg.precog_smc_route(t(emb), t(P), t(S), t(J, torch.int32), dm, dj, slot)
+    assert pg.precog_device_status()[0] == 0
+    rm, rj = oracle.smc_route(emb, P, S, J)
+    np.testing.assert_array_equal(dm.cpu().numpy(), rm)
+    np.testing.assert_array_equal(dj.cpu().numpy(), rj)
+    exp_slot = np.where(rj >= 0, rm * J_max + rj, -1)
+    np.testing.assert_array_equal(slot.cpu().numpy(), exp_slot)
+
+
+def test_consolidate_then_session_init(cuda_device):
+    """Deposit 300 chunk states (bf16, 24 layers of D=256, N=16) into 20 semantic slots
+    in order (some forgetting candidates, slot -1), compare the fp32 table with the
+    oracle's EMA, then initialise sessions from two slots and prefill 64 tokens."""
+    import torch
+    import paper_2608_02560_gb300 as pg
+    d = cuda_device
+    L, D, N, n, slots, alpha = 24, 256, 16, 300, 20, 0.2
+    rng = np.random.default_rng(3)
+    states = synth.device_normal_bank(n, L * D * N, 4, d)            # [n, elems] bf16
+    slot_np = rng.integers(-1, slots, size=n).astype(np.int64)
+    sem0 = rng.standard_normal((slots, L * D * N)).astype(np.float32) * 0.1
+    sem = torch.from_numpy(sem0).to(d)
+    pg.precog_smc_consolidate(sem, states, torch.from_numpy(slot_np).to(d), alpha)
+    assert pg.precog_device_status()[0] == 0
+    ref = oracle.smc_consolidate(sem0, to_np(states), slot_np, alpha)
+    got = to_np(sem)
+    for s in range(slots):
+        assert rel_err(got[s], ref[s]) < TOL_F32, s
+    # O(1) session initialisation: inject s_{m*, j*} and prefill (Sec. 5.3)
+    Tq, Q = 64, 2
+    ins = [synth.device_scan_inputs(Q * Tq, D, N, 5, l, d) for l in range(L)]
+    st = lambda k: torch.stack([i[k] for i in ins]).contiguous()
+    x, dt, B, C, A = st("x"), st("dt"), st("B"), st("C"), st("A")
+    idx = torch.tensor([3, 17], dtype=torch.int64, device=d)
+    h = torch.empty((Q, L, D, N), dtype=torch.float32, device=d)
+    pg.precog_prefill_from_state(pg.scan_inputs(x, dt, B, A, C, a_kind=pg.PRECOG_A_POWER), Q, Tq,
+                                 sem.view(slots, L, D, N), idx=idx, state_out=h)
+    assert pg.precog_device_status()[0] == 0
+    An = A[0].cpu().numpy()
+    for q, srow in enumerate((3, 17)):
+        for l in (0, 23):
+            sl = slice(q * Tq, (q + 1) * Tq)
+            ref_h, _ = oracle.rollout(to_np(x[l, sl]), to_np(dt[l, sl]), An, to_np(B[l, sl]),
+                                      h0=ref[srow].reshape(L, D, N)[l])
+            assert rel_err(to_np(h[q, l]), ref_h) < TOL_F32
