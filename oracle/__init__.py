@@ -21,6 +21,7 @@ module compiles it with gcc and marshals numpy arrays into it.
 * :func:`smc_route` -- two-level cluster routing of Sec. 5.1 (Eqs. smc-domain,
   smc-sub).
 * :func:`smc_consolidate` -- the semantic-state EMA of Sec. 5.3 (Eq. smc-ema).
+* :func:`scan_complex` -- the scan with the complex diagonal A of Eq. 1.
 """
 from __future__ import annotations
 
@@ -69,6 +70,10 @@ def _load():
         lib.oracle_trajectory.restype = ctypes.c_int
         lib.oracle_trajectory.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, p_i64,
                                           p_f64, p_f64, p_f64, p_f64, ctypes.c_int64, p_i64, p_f64]
+        lib.oracle_scan_complex.restype = ctypes.c_int
+        lib.oracle_scan_complex.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, p_i64,
+                                            p_f64, p_f64, p_f64, p_f64, p_f64, p_f64, p_f64, p_f64,
+                                            p_f64]
         lib.oracle_scores.restype = ctypes.c_int
         lib.oracle_scores.argtypes = [ctypes.c_int64, ctypes.c_int64, p_f64, ctypes.c_int64, p_f64,
                                       p_f64]
@@ -266,4 +271,27 @@ def smc_consolidate(semantic, states, slots, alpha):
             continue
         out[slot] = (1.0 - alpha) * out[slot] + alpha * h[c]
     return out
+
+
+def scan_complex(x, dt, A_re, A_im, B, offsets, C=None, h0=None, want_y=False):
+    """Complex-A scan of one layer (Eq. 1 with A = A_re + i A_im). h0 ``[n_chunks, D, N]``
+    complex. Returns ``(states complex128 [n_chunks, D, N], y float64 [T_tot, D] or None)``."""
+    lib = _load()
+    x, dt, A_re, A_im, B = _f64(x), _f64(dt), _f64(A_re), _f64(A_im), _f64(B)
+    C = _f64(C) if want_y else None
+    offsets = np.ascontiguousarray(np.asarray(offsets, dtype=np.int64))
+    D, N = A_re.shape
+    n_chunks = offsets.shape[0] - 1
+    T_tot = x.shape[0]
+    h0c = None if h0 is None else np.ascontiguousarray(np.asarray(h0, dtype=np.complex128))
+    states = np.zeros((n_chunks, D, N), dtype=np.complex128)
+    y = np.zeros((T_tot, D), dtype=np.float64) if want_y else None
+    p64, pi = ctypes.c_double, ctypes.c_int64
+    h0p = ctypes.POINTER(p64)() if h0c is None else h0c.ctypes.data_as(ctypes.POINTER(p64))
+    rc = lib.oracle_scan_complex(D, N, n_chunks, _ptr(offsets, pi), _ptr(x, p64), _ptr(dt, p64),
+                                 _ptr(A_re, p64), _ptr(A_im, p64), _ptr(B, p64), _ptr(C, p64), h0p,
+                                 states.ctypes.data_as(ctypes.POINTER(p64)), _ptr(y, p64))
+    if rc != 0:
+        raise ValueError(f"oracle_scan_complex rejected its arguments (rc={rc})")
+    return states, y
 

@@ -24,6 +24,7 @@
  *   stability premise |alpha(x)| < 1 of Appendix B.1; the oracle takes
  *   alpha = exp(dt*A) with A < 0 (equivalently exp(-dt*a) with rate a > 0).
  */
+#include <complex.h>
 #include <math.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -194,6 +195,53 @@ int oracle_trajectory(int64_t D, int64_t N, int64_t n_chunks, const int64_t *off
                     for (int64_t n = 0; n < N; ++n)
                         e[n] = h[n];
                     ++j;
+                }
+            }
+        }
+    }
+    return ORACLE_OK;
+}
+
+/*
+ * oracle_scan_complex: Eq. 1 with the complex diagonal A the paper prints
+ * (A_k = -softplus(a_k) + i*pi*k, Sec. 3) and a complex state h in C^N:
+ *   alpha = exp(dt * A[d,n])  (complex),   beta = B[t,n] * x[t,d] * dt[t,d]  (real)
+ *   h[d,n] = h[d,n] * alpha + beta,        y[t,d] = Re(sum_n C[t,n] * h[d,n])
+ * Reading: B and C stay real per (token, state index) as in the real scan, and
+ * the readout is the real part. A_re, A_im [D][N]; h0 and states_out are
+ * [n_chunks][D][N] double complex (re, im interleaved); h0 may be NULL.
+ */
+int oracle_scan_complex(int64_t D, int64_t N, int64_t n_chunks, const int64_t *offsets,
+                        const double *x, const double *dt, const double *A_re, const double *A_im,
+                        const double *B, const double *C, const double complex *h0,
+                        double complex *states_out, double *y_out)
+{
+    if (D <= 0 || N <= 0 || n_chunks < 0 || offsets == NULL || states_out == NULL)
+        return ORACLE_BAD_ARG;
+    if (y_out != NULL && C == NULL)
+        return ORACLE_BAD_ARG;
+    for (int64_t c = 0; c < n_chunks; ++c)
+        if (offsets[c] < 0 || offsets[c + 1] < offsets[c])
+            return ORACLE_BAD_ARG;
+    for (int64_t c = 0; c < n_chunks; ++c) {
+        for (int64_t d = 0; d < D; ++d) {
+            double complex *h = states_out + (c * D + d) * N;
+            for (int64_t n = 0; n < N; ++n)
+                h[n] = (h0 != NULL) ? h0[(c * D + d) * N + n] : 0.0;
+            for (int64_t t = offsets[c]; t < offsets[c + 1]; ++t) {
+                const double dt_td = dt[t * D + d];
+                const double x_td = x[t * D + d];
+                for (int64_t n = 0; n < N; ++n) {
+                    const double complex a = A_re[d * N + n] + I * A_im[d * N + n];
+                    const double complex alpha = cexp(dt_td * a);
+                    const double beta = B[t * N + n] * x_td * dt_td;
+                    h[n] = h[n] * alpha + beta;
+                }
+                if (y_out != NULL) {
+                    double y = 0.0;
+                    for (int64_t n = 0; n < N; ++n)
+                        y += C[t * N + n] * creal(h[n]);
+                    y_out[t * D + d] = y;
                 }
             }
         }

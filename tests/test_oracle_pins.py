@@ -418,3 +418,42 @@ def test_smc_consolidate_closed_form():
     out = oracle.smc_consolidate(s0, hs, [2, 0, 2, 0], 1.0)
     np.testing.assert_array_equal(out[2], hs[2])
     np.testing.assert_array_equal(out[0], hs[3])
+
+
+# ---------------------------------------------------------------- complex diagonal A
+
+
+def test_complex_scan_real_special_case():
+    """A_im = 0: the complex scan is the real scan (imaginary part stays exactly 0)."""
+    D, N = 3, 4
+    off = np.array([0, 9, 9, 30], dtype=np.int64)
+    x, dt, A, B, C = _rand_inputs(30, D, N, seed=5)
+    st, y = oracle.scan_complex(x, dt, A, np.zeros_like(A), B, off, C=C, want_y=True)
+    rs, ry = oracle.scan(x, dt, A, B, off, C=C, want_y=True)
+    np.testing.assert_allclose(st.real, rs, rtol=1e-13, atol=1e-14)
+    np.testing.assert_array_equal(st.imag, 0.0)
+    np.testing.assert_allclose(y, ry, rtol=1e-13, atol=1e-14)
+
+
+def test_complex_scan_theorem1_and_geometric_series():
+    """Theorem 1 holds for the complex recurrence (bit-identical sequential double), and
+    constant gates give the complex geometric series h_T = a^T h0 + b (1 - a^T)/(1 - a)."""
+    D, N = 2, 3
+    rng = np.random.default_rng(9)
+    A_re = -np.logaddexp(0.0, rng.standard_normal((D, N)))
+    A_im = np.pi * np.arange(N)[None, :].repeat(D, 0)          # i*pi*k of Eq. 1
+    x, dt, _, B, C = _rand_inputs(40, D, N, seed=10)
+    h0 = rng.standard_normal((1, D, N)) + 1j * rng.standard_normal((1, D, N))
+    full, yf = oracle.scan_complex(x, dt, A_re, A_im, B, [0, 40], C=C, h0=h0, want_y=True)
+    ctx, _ = oracle.scan_complex(x[:25], dt[:25], A_re, A_im, B[:25], [0, 25], h0=h0)
+    inj, yi = oracle.scan_complex(x[25:], dt[25:], A_re, A_im, B[25:], [0, 15], C=C[25:], h0=ctx,
+                                  want_y=True)
+    np.testing.assert_array_equal(full, inj)
+    np.testing.assert_array_equal(yf[25:], yi)
+    T, delta, xi = 30, 0.4, np.array([1.5, -0.5])
+    b = np.array([0.3, -1.0, 0.7])
+    hs, _ = oracle.scan_complex(np.tile(xi, (T, 1)), np.full((T, D), delta), A_re, A_im,
+                                np.tile(b, (T, 1)), [0, T], h0=h0)
+    a = np.exp(delta * (A_re + 1j * A_im))
+    beta = (delta * xi)[:, None] * b[None, :]
+    np.testing.assert_allclose(hs[0], a ** T * h0[0] + beta * (1 - a ** T) / (1 - a), rtol=1e-12)
