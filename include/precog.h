@@ -54,7 +54,8 @@ typedef enum precog_dtype {
 /* Structure of the diagonal state matrix A (see precog_scan_inputs). */
 typedef enum precog_a_kind {
     PRECOG_A_GENERAL = 0,  /* any A: one exponential per (channel, state index) */
-    PRECOG_A_POWER = 1     /* A[d,n] == (n+1)*A[d,0] exactly and A[d,0] <= 0 */
+    PRECOG_A_POWER = 1,    /* A[d,n] == (n+1)*A[d,0] exactly and A[d,0] <= 0 */
+    PRECOG_A_COMPLEX = 2   /* complex A: see precog_scan_inputs */
 } precog_a_kind;
 
 /* Device status bits reported by precog_device_status(). */
@@ -90,6 +91,14 @@ typedef enum precog_a_kind {
  * that alpha_n = r^(n+1) with r = exp(dt*A[d,0]): one exponential per (t, d).
  * The kernel verifies the statement per block of channels; where it is false
  * nothing is written for that block and PRECOG_DEV_BAD_A is flagged.
+ *
+ * PRECOG_A_COMPLEX selects the complex diagonal A that Eq. 1 prints
+ * (A_k = -softplus(a_k) + i*pi*k) with a complex state h in C^N: A points to
+ * [L][D][N] pairs (re, im) of fp32 (torch.complex64 layout); alpha =
+ * exp(dt*A) is complex, B and C stay real, y = Re(sum_n C[t,n] h[d,n]);
+ * states and banks hold (re, im) pairs per state index, [..][D][N][2]
+ * (complex64 for F32 state dtype, bf16 pairs for BF16). Accepted by
+ * precog_encode_chunks and precog_prefill_from_state (and k = 1 composition).
  */
 typedef struct precog_scan_inputs {
     int32_t n_layers;

@@ -27,7 +27,7 @@ LIB_PATH = os.path.join(_PKG, "libprecog.so")
 
 PRECOG_F32, PRECOG_BF16, PRECOG_F16 = 0, 1, 2
 PRECOG_OK = 0
-PRECOG_A_GENERAL, PRECOG_A_POWER = 0, 1
+PRECOG_A_GENERAL, PRECOG_A_POWER, PRECOG_A_COMPLEX = 0, 1, 2
 PRECOG_DEV_BAD_OFFSETS, PRECOG_DEV_BAD_INDEX, PRECOG_DEV_TIMEOUT, PRECOG_DEV_BAD_A = 0x1, 0x2, 0x4, 0x8
 STATUS_NAMES = {0: "PRECOG_OK", 1: "PRECOG_ERR_INVALID_ARG", 2: "PRECOG_ERR_UNSUPPORTED",
                 3: "PRECOG_ERR_CUDA", 4: "PRECOG_ERR_TIMEOUT", 5: "PRECOG_ERR_DEVICE"}
@@ -108,7 +108,9 @@ def _check(status: int):
 
 def _dtype_code(t) -> int:
     import torch
-    m = {torch.float32: PRECOG_F32, torch.bfloat16: PRECOG_BF16, torch.float16: PRECOG_F16}
+    # complex64 state/bank buffers are (re, im) fp32 pairs: the F32 storage code
+    m = {torch.float32: PRECOG_F32, torch.bfloat16: PRECOG_BF16, torch.float16: PRECOG_F16,
+         torch.complex64: PRECOG_F32}
     if t.dtype not in m:
         raise TypeError(f"unsupported dtype {t.dtype}")
     return m[t.dtype]
@@ -135,7 +137,8 @@ def scan_inputs(x, dt, B, A, C=None, a_kind: int = PRECOG_A_GENERAL) -> ScanInpu
     """Describe x, dt ``[L, T, D]`` (or ``[T, D]``), B, C ``[L, T, N]``, A ``[L, D, N]``.
 
     ``a_kind=PRECOG_A_POWER`` states that A[d, n] == (n + 1) * A[d, 0] <= 0 (verified on
-    the device); it selects the one-exponential update forms."""
+    the device); it selects the one-exponential update forms. ``a_kind=PRECOG_A_COMPLEX``
+    takes a complex64 A (Eq. 1's complex diagonal) and complex states."""
     if x.dim() == 2:
         x, dt, B = x.unsqueeze(0), dt.unsqueeze(0), B.unsqueeze(0)
         C = None if C is None else C.unsqueeze(0)
@@ -146,7 +149,10 @@ def scan_inputs(x, dt, B, A, C=None, a_kind: int = PRECOG_A_GENERAL) -> ScanInpu
     if dt.shape != x.shape or B.shape != (L, T, N) or (C is not None and C.shape != B.shape):
         raise ValueError("x/dt/B/C shapes disagree")
     import torch
-    if A.shape != (L, D, N) or A.dtype != torch.float32:
+    if a_kind == PRECOG_A_COMPLEX:
+        if A.shape != (L, D, N) or A.dtype != torch.complex64:
+            raise ValueError("complex A must be complex64 [L, D, N]")
+    elif A.shape != (L, D, N) or A.dtype != torch.float32:
         raise ValueError("A must be float32 [L, D, N]")
     s = ScanInputs()
     # the struct holds raw device pointers: keep the tensors alive as long as it lives

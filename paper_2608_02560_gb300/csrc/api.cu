@@ -49,8 +49,9 @@ precog_status check_scan_inputs(const precog_scan_inputs *in, int64_t rows, bool
     if (in->n_layers < 1) return fail(PRECOG_ERR_INVALID_ARG, "n_layers must be >= 1");
     if (in->N != 16) return fail(PRECOG_ERR_UNSUPPORTED, "N=%d: only N=16 is implemented", in->N);
     if (in->D < 1) return fail(PRECOG_ERR_INVALID_ARG, "D must be >= 1");
-    if (in->a_kind != PRECOG_A_GENERAL && in->a_kind != PRECOG_A_POWER)
-        return fail(PRECOG_ERR_INVALID_ARG, "a_kind must be PRECOG_A_GENERAL or PRECOG_A_POWER");
+    if (in->a_kind != PRECOG_A_GENERAL && in->a_kind != PRECOG_A_POWER &&
+        in->a_kind != PRECOG_A_COMPLEX)
+        return fail(PRECOG_ERR_INVALID_ARG, "a_kind must be PRECOG_A_GENERAL, _POWER or _COMPLEX");
     if (in->in_dtype != PRECOG_F32 && in->in_dtype != PRECOG_BF16)
         return fail(PRECOG_ERR_UNSUPPORTED, "in_dtype must be PRECOG_F32 or PRECOG_BF16");
     const int sz = dtype_size(in->in_dtype);
@@ -146,7 +147,9 @@ precog_status precog_encode_chunks(const precog_scan_inputs *in, const int64_t *
     p.layer0 = states_out ? layer0 : 0;
     p.y = y_out;
     p.y_dtype = y_dtype;
-    cudaError_t e = precog::launch_scan(p, static_cast<cudaStream_t>(stream));
+    cudaError_t e = in->a_kind == PRECOG_A_COMPLEX
+                        ? precog::launch_scan_complex(p, static_cast<cudaStream_t>(stream))
+                        : precog::launch_scan(p, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
     return ok();
 }
@@ -191,7 +194,9 @@ precog_status precog_prefill_from_state(const precog_scan_inputs *in, int32_t n_
     p.layer0 = layer0;
     p.y = y_out;
     p.y_dtype = y_dtype;
-    cudaError_t e = precog::launch_scan(p, static_cast<cudaStream_t>(stream));
+    cudaError_t e = in->a_kind == PRECOG_A_COMPLEX
+                        ? precog::launch_scan_complex(p, static_cast<cudaStream_t>(stream))
+                        : precog::launch_scan(p, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "prefill launch");
     return ok();
 }
@@ -206,6 +211,8 @@ precog_status precog_encode_trajectory(const precog_scan_inputs *in, const int64
     if (s != PRECOG_OK) return s;
     if (n_chunks < 0) return fail(PRECOG_ERR_INVALID_ARG, "n_chunks must be >= 0");
     if (stride < 1) return fail(PRECOG_ERR_INVALID_ARG, "stride must be >= 1");
+    if (in->a_kind == PRECOG_A_COMPLEX)
+        return fail(PRECOG_ERR_UNSUPPORTED, "trajectories of a complex-A scan are not implemented");
     if (d_offsets == nullptr || d_entry_offsets == nullptr)
         return fail(PRECOG_ERR_INVALID_ARG, "d_offsets and d_entry_offsets must be non-NULL");
     if (traj_out == nullptr || !state_dtype_ok(traj_dtype) || !aligned16(traj_out))
@@ -235,6 +242,8 @@ precog_status precog_prefill_composed(const precog_scan_inputs *in, int32_t n_qu
                                      int32_t state_dtype, void *stream) {
     if (k < 1 || k > 8) return fail(PRECOG_ERR_UNSUPPORTED, "k must be in [1, 8]");
     if (d_idx == nullptr) return fail(PRECOG_ERR_INVALID_ARG, "d_idx is NULL");
+    if (in != nullptr && in->a_kind == PRECOG_A_COMPLEX && k > 1)
+        return fail(PRECOG_ERR_UNSUPPORTED, "composition of complex states is not implemented");
     if (k > 1 && d_score == nullptr) return fail(PRECOG_ERR_INVALID_ARG, "d_score is NULL");
     if (!(temperature > 0.f)) return fail(PRECOG_ERR_INVALID_ARG, "temperature must be > 0");
     if (k == 1)
@@ -412,10 +421,12 @@ precog_status precog_device_status(void *stream, uint32_t *bits_out) {
     if (e != cudaSuccess) return cuda_fail(e, "read scan status");
     e = precog::retrieve_status_word_read_clear(&b);
     if (e != cudaSuccess) return cuda_fail(e, "read retrieve status");
-    uint32_t c = 0;
+    uint32_t c = 0, z = 0;
     e = precog::smc_status_word_read_clear(&c);
     if (e != cudaSuccess) return cuda_fail(e, "read smc status");
-    *bits_out = a | b | c;
+    e = precog::scan_complex_status_word_read_clear(&z);
+    if (e != cudaSuccess) return cuda_fail(e, "read complex scan status");
+    *bits_out = a | b | c | z;
     if (*bits_out == 0) return ok();
     if (*bits_out & PRECOG_DEV_TIMEOUT)
         return fail(PRECOG_ERR_TIMEOUT, "a device-side wait gave up (bits 0x%x)", *bits_out);

@@ -87,6 +87,11 @@ cudaError_t launch_retrieve_tc_topk(const RetrieveParams &p, int grid, cudaStrea
 cudaError_t launch_retrieve(const RetrieveParams &p, cudaStream_t stream);
 cudaError_t retrieve_status_word_read_clear(uint32_t *bits);
 
+// Complex diagonal A (scan_complex.cu): A is [L][D][N] (re, im) pairs, states
+// [..][D][N] (re, im) pairs.
+cudaError_t launch_scan_complex(const ScanParams &p, cudaStream_t stream);
+cudaError_t scan_complex_status_word_read_clear(uint32_t *bits);
+
 // SMC primitives (smc.cu)
 cudaError_t launch_smc_route(const void *emb, int dtype, int64_t n, int dim, const void *dom, int M,
                              const void *sub, int J_max, const int32_t *J, int32_t *out_m,

@@ -1,0 +1,172 @@
+// The scan with the complex diagonal A that Eq. 1 prints (A_k = -softplus(a_k)
+// + i*pi*k, h in C^N): alpha = exp(dt * A) = e^(dt*A_re) (cos + i sin)(dt*A_im),
+// beta = B * x * dt real, y = Re(sum_n C_n h_n). Correctness-first: one thread
+// per channel with its 16 complex states in registers, inputs read straight
+// from global memory (coalesced across the channels of a block; B and C rows
+// are shared by the block and served from L1). One SFU exponential and one
+// sine/cosine pair per (token, channel, state index); the phase dt * A_im is
+// formed exactly as a two-float product (fma error term) and reduced to
+// [-pi, pi] by Cody-Waite with 2*pi split into two floats before the SFU
+// sine and cosine.
+#include <type_traits>
+
+#include "../../include/precog.h"
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace precog {
+namespace {
+
+__device__ uint32_t g_scan_complex_status;
+
+constexpr int kN = 16;
+constexpr int kBlock = 128;
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kInv2Pi = 0.15915494309189535f;
+constexpr float k2PiHi = 6.28318548202514648f;     // fp32 nearest to 2*pi
+constexpr float k2PiLo = -1.7484556000744487e-07f; // 2*pi - k2PiHi
+
+__device__ __forceinline__ void sincos_reduced(float hi, float lo, float &s, float &c) {
+    const float k = rintf(hi * kInv2Pi);
+    float r = fmaf(-k, k2PiHi, hi);
+    r = fmaf(-k, k2PiLo, r);
+    r += lo;
+    asm("sin.approx.ftz.f32 %0, %1;" : "=f"(s) : "f"(r));
+    asm("cos.approx.ftz.f32 %0, %1;" : "=f"(c) : "f"(r));
+}
+
+template <typename TIn>
+__device__ __forceinline__ float ld(const TIn *p) {
+    return to_f32(__ldg(p));
+}
+
+template <typename TIn, bool HAS_Y, bool HAS_H0>
+__global__ void __launch_bounds__(kBlock)
+    scan_complex_kernel(const ScanParams p, const int cblocks) {
+    int64_t item = blockIdx.x;
+    const int cb = static_cast<int>(item % cblocks);
+    item /= cblocks;
+    const int64_t chunk = item % p.n_chunks;
+    const int layer = static_cast<int>(item / p.n_chunks);
+    const int d = cb * kBlock + threadIdx.x;
+    const int D = p.D;
+    int64_t start, len;
+    if (p.use_fixed) {
+        start = chunk * p.fixed_len;
+        len = p.fixed_len;
+    } else {
+        start = p.offsets[chunk];
+        const int64_t end = p.offsets[chunk + 1];
+        if (start < 0 || end < start || end > p.T_tot) {
+            if (threadIdx.x == 0) atomicOr(&g_scan_complex_status, PRECOG_DEV_BAD_OFFSETS);
+            return;
+        }
+        len = end - start;
+    }
+    if (d >= D) return;
+    const TIn *xl = static_cast<const TIn *>(p.x) + layer * p.ls_xd;
+    const TIn *dtl = static_cast<const TIn *>(p.dt) + layer * p.ls_xd;
+    const TIn *Bl = static_cast<const TIn *>(p.B) + layer * p.ls_bc;
+    const TIn *Cl = HAS_Y ? static_cast<const TIn *>(p.C) + layer * p.ls_bc : nullptr;
+    const float2 *Al = reinterpret_cast<const float2 *>(p.A) + (static_cast<int64_t>(layer) * D + d) * kN;
+
+    float ar[kN], ai[kN], hr[kN], hi[kN];
+#pragma unroll
+    for (int n = 0; n < kN; ++n) {
+        const float2 a = Al[n];
+        ar[n] = a.x * kLog2e;
+        ai[n] = a.y;
+        hr[n] = 0.f;
+        hi[n] = 0.f;
+    }
+    if constexpr (HAS_H0) {
+        const int64_t row = p.idx ? p.idx[chunk] : chunk;
+        if (row >= 0 && row < p.bank_entries) {
+            const int64_t off = ((row * p.L_bank + p.layer0 + layer) * static_cast<int64_t>(D) + d) * kN;
+#pragma unroll
+            for (int n = 0; n < kN; ++n) {
+                if (p.bank_dtype == PRECOG_F32) {
+                    const float2 v = reinterpret_cast<const float2 *>(p.bank)[off + n];
+                    hr[n] = v.x;
+                    hi[n] = v.y;
+                } else {
+                    const __nv_bfloat162 v = reinterpret_cast<const __nv_bfloat162 *>(p.bank)[off + n];
+                    hr[n] = __low2float(v);
+                    hi[n] = __high2float(v);
+                }
+            }
+        } else if (!(p.idx && row == -1) && threadIdx.x == 0) {
+            atomicOr(&g_scan_complex_status, PRECOG_DEV_BAD_INDEX);
+        }
+    }
+    for (int64_t t = start; t < start + len; ++t) {
+        const float xv = ld(xl + t * D + d);
+        const float dv = ld(dtl + t * D + d);
+        const float u = dv * xv;
+        float y = 0.f;
+#pragma unroll
+        for (int n = 0; n < kN; ++n) {
+            const float mag = ex2(dv * ar[n]);
+            const float th = dv * ai[n];
+            const float tl = fmaf(dv, ai[n], -th);   // exact error of the product
+            float s, c;
+            sincos_reduced(th, tl, s, c);
+            const float are = mag * c, aim = mag * s;
+            const float nr = fmaf(are, hr[n], fmaf(-aim, hi[n], u * ld(Bl + t * kN + n)));
+            const float ni = fmaf(are, hi[n], aim * hr[n]);
+            hr[n] = nr;
+            hi[n] = ni;
+            if constexpr (HAS_Y) y = fmaf(ld(Cl + t * kN + n), nr, y);
+        }
+        if constexpr (HAS_Y) {
+            const int64_t yo = (static_cast<int64_t>(layer) * p.T_tot + t) * D + d;
+            if (p.y_dtype == PRECOG_F32) static_cast<float *>(p.y)[yo] = y;
+            else static_cast<__nv_bfloat16 *>(p.y)[yo] = __float2bfloat16_rn(y);
+        }
+    }
+    if (p.states) {
+        const int64_t off = ((chunk * p.L_out + p.layer0 + layer) * static_cast<int64_t>(D) + d) * kN;
+#pragma unroll
+        for (int n = 0; n < kN; ++n) {
+            if (p.state_dtype == PRECOG_F32)
+                reinterpret_cast<float2 *>(p.states)[off + n] = make_float2(hr[n], hi[n]);
+            else
+                reinterpret_cast<__nv_bfloat162 *>(p.states)[off + n] = __floats2bfloat162_rn(hr[n], hi[n]);
+        }
+    }
+}
+
+template <typename TIn, bool HAS_Y, bool HAS_H0>
+cudaError_t launch_c(const ScanParams &p, cudaStream_t stream) {
+    const int cblocks = (p.D + kBlock - 1) / kBlock;
+    const int64_t items = static_cast<int64_t>(p.n_layers) * p.n_chunks * cblocks;
+    if (items == 0) return cudaSuccess;
+    if (items > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+    scan_complex_kernel<TIn, HAS_Y, HAS_H0><<<static_cast<unsigned>(items), kBlock, 0, stream>>>(p, cblocks);
+    cudaError_t e = cudaGetLastError();
+    if (e == cudaSuccess) count_launches(1);
+    return e;
+}
+
+template <typename TIn>
+cudaError_t launch_in(const ScanParams &p, cudaStream_t stream) {
+    const bool y = p.y != nullptr, h0 = p.bank != nullptr;
+    if (y) return h0 ? launch_c<TIn, true, true>(p, stream) : launch_c<TIn, true, false>(p, stream);
+    return h0 ? launch_c<TIn, false, true>(p, stream) : launch_c<TIn, false, false>(p, stream);
+}
+
+}  // namespace
+
+cudaError_t launch_scan_complex(const ScanParams &p, cudaStream_t stream) {
+    if (p.in_dtype == PRECOG_F32) return launch_in<float>(p, stream);
+    return launch_in<__nv_bfloat16>(p, stream);
+}
+
+cudaError_t scan_complex_status_word_read_clear(uint32_t *bits) {
+    uint32_t zero = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(bits, g_scan_complex_status, sizeof(uint32_t));
+    if (e != cudaSuccess) return e;
+    return cudaMemcpyToSymbol(g_scan_complex_status, &zero, sizeof(uint32_t));
+}
+
+}  // namespace precog

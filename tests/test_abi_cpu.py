@@ -68,12 +68,24 @@ def _encode(lib, s, offsets=FAKE, n_chunks=4, T_tot=64, states=FAKE, sdt=0, laye
 @pytest.mark.parametrize("change,expect", [
     ({"N": 8}, 2), ({"D": 0}, 1), ({"D": 12}, 2), ({"in_dtype": 2}, 2), ({"x": 0}, 1),
     ({"A": FAKE + 4}, 1), ({"n_layers": 0}, 1), ({"n_layers": 2, "layer_stride_xd": 10}, 1),
-    ({"a_kind": 2}, 1), ({"a_kind": -1}, 1),
+    ({"a_kind": 3}, 1), ({"a_kind": -1}, 1),
 ])
 def test_encode_rejects_bad_inputs(lib, change, expect):
     import paper_2608_02560_gb300 as pg
     assert _encode(lib, _inputs(pg, **change)) == expect
     assert lib.precog_last_error() != b""
+
+
+def test_complex_A_forms_without_a_kernel_are_rejected(lib):
+    """Trajectories and k > 1 composition of complex states are refused as unsupported
+    before any launch."""
+    import paper_2608_02560_gb300 as pg
+    s = _inputs(pg, a_kind=pg.PRECOG_A_COMPLEX)
+    st = lib.precog_encode_trajectory(ctypes.byref(s), FAKE, 4, 64, 8, FAKE, FAKE, 0, 0, 1, None)
+    assert st == 2 and b"complex" in lib.precog_last_error()
+    st = lib.precog_prefill_composed(ctypes.byref(s), 2, 32, FAKE, 0, 10, 1, 0, 3, FAKE, FAKE,
+                                     1.0, None, 0, FAKE, 0, None)
+    assert st == 2 and b"complex" in lib.precog_last_error()
 
 
 def test_encode_rejects_bad_call_arguments(lib):

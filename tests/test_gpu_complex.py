@@ -1,0 +1,181 @@
+"""GPU parity of the complex-diagonal-A scan (Eq. 1 with A_k = -softplus(a_k) + i*pi*k and
+h in C^N; real B and C, readout y = Re sum_n C_n h_n) against the oracle's complex rollout:
+encode with state capture and readout, ragged and empty chunks, bf16 storage, prefill
+from an injected complex state (Theorem 1), and the real special case A_im = 0."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from tests._util import TOL_BF16, TOL_F32, rel_err, rel_err_stored, to_np
+
+pytestmark = pytest.mark.gpu
+
+
+def _pg():
+    import paper_2608_02560_gb300 as pg
+    return pg
+
+
+def _complex_A(D, N, seed):
+    """The paper's parameterisation: real part -softplus(a), imaginary part pi * k."""
+    rng = np.random.default_rng(seed)
+    a = rng.standard_normal((D, N))
+    re = -synth.softplus_np(a)
+    im = np.broadcast_to(np.pi * np.arange(N), (D, N))
+    return (re + 1j * im).astype(np.complex64)
+
+
+def _cplx_err(got, ref):
+    got = np.asarray(got, dtype=np.complex128)
+    return float(np.max(np.abs(got - ref)) / max(np.max(np.abs(ref)), 1e-30))
+
+
+def _t(a, d, dtype=None):
+    import torch
+    t = torch.from_numpy(np.ascontiguousarray(a)).to(d)
+    return t if dtype is None else t.to(dtype)
+
+
+def _encode(pg, d, x, dt, B, C, A, offsets, state_dtype="complex64", with_y=True, in_dtype=None):
+    import torch
+    T, D = x.shape
+    N = B.shape[1]
+    n = len(offsets) - 1
+    ins = pg.scan_inputs(_t(x, d, in_dtype), _t(dt, d, in_dtype), _t(B, d, in_dtype),
+                         _t(A, d), _t(C, d, in_dtype) if with_y else None, a_kind=pg.PRECOG_A_COMPLEX)
+    if state_dtype == "complex64":
+        st = torch.full((n, 1, D, N), float("nan"), dtype=torch.complex64, device=d)
+    else:
+        st = torch.full((n, 1, D, N, 2), float("nan"), dtype=torch.bfloat16, device=d)
+    y = torch.full((1, T, D), float("nan"), dtype=in_dtype or torch.float32, device=d) if with_y else None
+    pg.precog_encode_chunks(ins, _t(offsets, d), T, states_out=st, y_out=y)
+    assert pg.precog_device_status()[0] == 0
+    if state_dtype == "complex64":
+        hs = st[:, 0].cpu().numpy().astype(np.complex128)
+    else:
+        f = st[:, 0].float().cpu().numpy().astype(np.float64)
+        hs = f[..., 0] + 1j * f[..., 1]
+    return hs, (None if y is None else to_np(y[0]))
+
+
+@pytest.mark.parametrize("D,offsets", [
+    (64, [0, 1, 17, 17, 160, 400]),               # a one-token, an empty and ragged chunks
+    (256, [0, 512, 1024]),
+    (200, [0, 3, 700]),                           # D not a multiple of the 128-channel block
+])
+def test_complex_encode_fp32(cuda_device, D, offsets):
+    pg = _pg()
+    T = offsets[-1]
+    x, dt, _, B, C = synth.host_scan_inputs(T, D, 16, seed=D + T)
+    A = _complex_A(D, 16, D)
+    hs, y = _encode(pg, cuda_device, x, dt, B, C, A, np.array(offsets, np.int64))
+    ref_h, ref_y = oracle.scan_complex(x, dt, A.real, A.imag, B, offsets, C=C, want_y=True)
+    assert _cplx_err(hs, ref_h) < TOL_F32
+    assert rel_err(y, ref_y) < TOL_F32
+    empty = [c for c in range(len(offsets) - 1) if offsets[c] == offsets[c + 1]]
+    for c in empty:
+        assert np.all(hs[c] == 0)
+
+
+def test_complex_encode_bf16_inputs_and_states(cuda_device):
+    import torch
+    pg = _pg()
+    D, T = 128, 1500
+    offsets = np.array([0, 300, 301, 1100, 1500], np.int64)
+    x, dt, _, B, C = synth.host_scan_inputs(T, D, 16, seed=5)
+    # the oracle sees the bf16-rounded values the kernel reads
+    rnd = lambda a: torch.from_numpy(a).to(torch.bfloat16).float().numpy()
+    x, dt, B, C = rnd(x), rnd(dt), rnd(B), rnd(C)
+    A = _complex_A(D, 16, 6)
+    hs, y = _encode(pg, cuda_device, x, dt, B, C, A, offsets, state_dtype="bf16",
+                    in_dtype=torch.bfloat16)
+    ref_h, ref_y = oracle.scan_complex(x, dt, A.real, A.imag, B, offsets, C=C, want_y=True)
+    # each stored component carries at most half a bf16 ulp on top of the fp32 error
+    assert rel_err_stored(hs.real, ref_h.real) < TOL_BF16
+    assert rel_err_stored(hs.imag, ref_h.imag) < TOL_BF16
+    assert rel_err_stored(y, ref_y) < TOL_BF16
+
+
+def test_complex_real_special_case_matches_real_scan(cuda_device):
+    """A_im = 0: the complex kernel's real part equals the real kernel's state and the
+    imaginary part stays exactly zero."""
+    import torch
+    pg = _pg()
+    d = cuda_device
+    D, T = 128, 900
+    offsets = np.array([0, 450, 900], np.int64)
+    x, dt, Ar, B, C = synth.host_scan_inputs(T, D, 16, seed=9)
+    A = (Ar.astype(np.float64) + 0j).astype(np.complex64)
+    hs, y = _encode(pg, d, x, dt, B, C, A, offsets)
+    assert np.all(hs.imag == 0)
+    st = torch.empty((2, 1, D, 16), dtype=torch.float32, device=d)
+    yr = torch.empty((1, T, D), dtype=torch.float32, device=d)
+    pg.precog_encode_chunks(pg.scan_inputs(_t(x, d), _t(dt, d), _t(B, d), _t(Ar, d), _t(C, d)),
+                            _t(offsets, d), T, states_out=st, y_out=yr)
+    assert rel_err(hs.real, st[:, 0].cpu().numpy().astype(np.float64)) < 1e-6
+    assert rel_err(y, to_np(yr[0])) < 1e-6
+
+
+@pytest.mark.parametrize("bank_kind", ["complex64", "bf16"])
+def test_complex_prefill_theorem1(cuda_device, bank_kind):
+    """S(h0, c (+) q) = S(S(h0, c), q): encode chunk c, inject its complex state, prefill q;
+    compare with the oracle's rollout of c (+) q, and a missing row (-1) starts from zero."""
+    import torch
+    pg = _pg()
+    d = cuda_device
+    D, Tc, Tq, Q = 64, 300, 50, 3
+    x, dt, _, B, C = synth.host_scan_inputs(Q * (Tc + Tq), D, 16, seed=21)
+    A = _complex_A(D, 16, 22)
+    xc, dtc, Bc, Cc = x[:Q * Tc], dt[:Q * Tc], B[:Q * Tc], C[:Q * Tc]
+    xq, dtq, Bq, Cq = x[Q * Tc:], dt[Q * Tc:], B[Q * Tc:], C[Q * Tc:]
+    offs = np.arange(Q + 1, dtype=np.int64) * Tc
+    hs, _ = _encode(pg, d, xc, dtc, Bc, Cc, A, offs, with_y=False)
+    if bank_kind == "complex64":
+        bank = torch.from_numpy(hs.astype(np.complex64)).to(d).view(Q, 1, D, 16)
+        h_inj = hs
+    else:
+        pair = np.stack([hs.real, hs.imag], axis=-1).astype(np.float32)
+        bank = torch.from_numpy(pair).to(d, torch.bfloat16).view(Q, 1, D, 16, 2)
+        f = bank[:, 0].float().cpu().numpy().astype(np.float64)
+        h_inj = f[..., 0] + 1j * f[..., 1]
+    idx = torch.tensor([2, -1, 0], dtype=torch.int64, device=d)
+    y = torch.empty((1, Q * Tq, D), dtype=torch.float32, device=d)
+    h = torch.empty((Q, 1, D, 16), dtype=torch.complex64, device=d)
+    ins = pg.scan_inputs(_t(xq, d), _t(dtq, d), _t(Bq, d), _t(A, d), _t(Cq, d),
+                         a_kind=pg.PRECOG_A_COMPLEX)
+    pg.precog_prefill_from_state(ins, Q, Tq, bank, idx=idx, y_out=y, state_out=h)
+    assert pg.precog_device_status()[0] == 0
+    for q, row in enumerate([2, -1, 0]):
+        h0 = np.zeros((1, D, 16), np.complex128) if row < 0 else h_inj[row][None]
+        sl = slice(q * Tq, (q + 1) * Tq)
+        ref_h, ref_y = oracle.scan_complex(xq[sl], dtq[sl], A.real, A.imag, Bq[sl], [0, Tq],
+                                           C=Cq[sl], h0=h0, want_y=True)
+        assert _cplx_err(h[q, 0].cpu().numpy(), ref_h[0]) < TOL_F32
+        assert rel_err(to_np(y[0, sl]), ref_y) < TOL_F32
+        if row >= 0 and bank_kind == "complex64":
+            # the whole concatenation from zero (Theorem 1)
+            cat = lambda a, b: np.concatenate([a[row * Tc:(row + 1) * Tc], b[sl]])
+            full, _ = oracle.scan_complex(cat(xc, xq), cat(dtc, dtq), A.real, A.imag, cat(Bc, Bq),
+                                          [0, Tc + Tq])
+            assert _cplx_err(h[q, 0].cpu().numpy(), full[0]) < TOL_F32
+
+
+def test_complex_unsupported_forms_are_rejected(cuda_device):
+    import torch
+    pg = _pg()
+    d = cuda_device
+    D, T = 64, 8
+    x, dt, _, B, C = synth.host_scan_inputs(T, D, 16, seed=1)
+    A = _complex_A(D, 16, 2)
+    ins = pg.scan_inputs(_t(x, d), _t(dt, d), _t(B, d), _t(A, d), _t(C, d), a_kind=pg.PRECOG_A_COMPLEX)
+    offs = _t(np.array([0, T], np.int64), d)
+    with pytest.raises(pg.PrecogError):
+        pg.precog_encode_trajectory(ins, offs, T, 4, _t(np.array([0, 2], np.int64), d),
+                                    torch.empty((2, 1, D, 16), dtype=torch.complex64, device=d))
+    bank = torch.zeros((4, 1, D, 16), dtype=torch.complex64, device=d)
+    rows = torch.zeros((1, 2), dtype=torch.int64, device=d)
+    sc = torch.zeros((1, 2), dtype=torch.float32, device=d)
+    with pytest.raises(pg.PrecogError):
+        pg.precog_prefill_composed(ins, 1, T, bank, rows, sc, 2,
+                                   state_out=torch.empty((1, 1, D, 16), dtype=torch.complex64, device=d))
