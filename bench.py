@@ -59,6 +59,8 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-latency", action="store_true")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="skip the measurements of the extension rows (top-k, trajectory, complex A, SMC)")
     ap.add_argument("--case", choices=["full", "scan-small", "retrieve-small", "prefill-small"],
                     default="full",
                     help="small single-kernel cases (a few GB) used for profiler captures")
@@ -250,6 +252,101 @@ def run_case(args):
         sys.exit(1)
 
 
+# ------------------------------------------------------------------------------ extension rows
+
+
+def measure_extensions(pg, synth, torch, dev, layer_in, off, T, n_chunks, index, qbank, query_batch, hbm):
+    """Times the extension rows on the resident paper-shaped buffers (a few seconds):
+    top-k retrieval and composed prefill (Sec. 4.4), K-dial trajectory capture (Sec. 5.2),
+    the complex-A scan (Eq. 1's complex diagonal) and the SMC routing / EMA kernels (Sec. 5).
+    Each entry: median ms over a few launches (L2 flushed before each), algorithmic bytes
+    (or flops) of one launch and the fraction of the measured peak they reach."""
+    import numpy as np
+    D, N = layer_in["x"].shape[1], layer_in["B"].shape[1]
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+
+    def timed(fn, iters=5):
+        fn()
+        ts = []
+        for _ in range(iters):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            b.record()
+            b.synchronize()
+            ts.append(a.elapsed_time(b))
+        ts.sort()
+        return ts[len(ts) // 2]
+
+    def hbm_row(ms, nbytes, **kw):
+        gbs = nbytes / (ms * 1e-3) / 1e9
+        return dict(ms=ms, algorithmic_bytes=nbytes, achieved_gbs=gbs, frac_hbm=gbs / hbm, **kw)
+
+    out = {}
+    in_bytes = T * (2 * D + N) * 2
+    # f2: trajectory, one state every 1000 tokens of each 3000-token chunk (K = 3)
+    stride = 1000
+    lens = (off[1:] - off[:-1]).cpu().numpy()
+    eo_np = np.concatenate([[0], np.cumsum((lens + stride - 1) // stride)]).astype(np.int64)
+    eo = torch.from_numpy(eo_np).to(dev)
+    traj = torch.empty((int(eo_np[-1]), 1, D, N), dtype=torch.bfloat16, device=dev)
+    si = pg.scan_inputs(layer_in["x"], layer_in["dt"], layer_in["B"], layer_in["A"], a_kind=pg.PRECOG_A_POWER)
+    ms = timed(lambda: pg.precog_encode_trajectory(si, off, T, stride, eo, traj), 3)
+    out["trajectory_stride1000"] = hbm_row(ms, in_bytes + traj.numel() * 2, entries=int(eo_np[-1]),
+                                           tokens_per_s=T / (ms * 1e-3))
+    del traj
+    # f3: complex A, paper parameterisation (real part -(n+1), imaginary part pi*n)
+    A = torch.complex(layer_in["A"], (math.pi * torch.arange(N, device=dev, dtype=torch.float32)).expand(D, N))
+    A = A.contiguous()
+    sc = pg.scan_inputs(layer_in["x"], layer_in["dt"], layer_in["B"], A, a_kind=pg.PRECOG_A_COMPLEX)
+    cst = torch.empty((n_chunks, 1, D, N, 2), dtype=torch.bfloat16, device=dev)
+    ms = timed(lambda: pg.precog_encode_chunks(sc, off, T, states_out=cst), 3)
+    out["complex_A_encode"] = hbm_row(ms, in_bytes + cst.numel() * 2, tokens_per_s=T / (ms * 1e-3),
+                                      bound="alu (SFU: exp, sin, cos per state update)")
+    del cst
+    # f1: top-3 retrieval over the 1M index and the composed 24-layer prefill
+    M, dim = index.shape
+    for nq in (1, 256):
+        b = query_batch(nq, 4242 + nq)
+        k = 3
+        ti = torch.empty((nq, k), dtype=torch.int64, device=dev)
+        ts_ = torch.empty((nq, k), dtype=torch.float32, device=dev)
+        ws = torch.empty(pg.precog_retrieve_topk_workspace_size(M, dim, nq) + 16, dtype=torch.uint8, device=dev)
+        ms_r = timed(lambda: pg.precog_retrieve_topk(index, b["q"], k, ti, ts_, workspace=ws))
+        Tq = b["x"].shape[1] // nq
+        ms_c = timed(lambda: pg.precog_prefill_composed(b["in"], nq, Tq, qbank, ti, ts_, k,
+                                                        y_out=b["y"], state_out=b["h"]))
+        row = hbm_row(ms_r, M * dim * 2, k=k, planted_first=bool(torch.equal(ti[:, 0], b["rows"])))
+        if nq > 1:
+            row["tflops"] = 2.0 * nq * M * dim / (ms_r * 1e-3) / 1e12
+        out[f"topk_retrieve_q{nq}"] = row
+        L = qbank.shape[1]
+        cb = nq * k * L * D * N * 2 + b["x"].numel() * 4 + b["B"].numel() * 4 + b["y"].numel() * 2 + b["h"].numel() * 2
+        out[f"composed_prefill_q{nq}_k3"] = hbm_row(ms_c, cb)
+        del b, ws
+    # f4: SMC routing of 4096 chunk embeddings into 16 domains x 64 sub-clusters, and the
+    # EMA of 4096 captured 24-layer states into 64 semantic slots
+    n_emb, Md, J = 4096, 16, 64
+    emb = index[:n_emb]
+    dom = index[n_emb:n_emb + Md].contiguous()
+    sub = index[n_emb + Md:n_emb + Md + Md * J].contiguous().view(Md, J, dim)
+    Jt = torch.full((Md,), J, dtype=torch.int32, device=dev)
+    om = torch.empty(n_emb, dtype=torch.int32, device=dev)
+    oj = torch.empty(n_emb, dtype=torch.int32, device=dev)
+    os_ = torch.empty(n_emb, dtype=torch.int64, device=dev)
+    ms = timed(lambda: pg.precog_smc_route(emb, dom, sub, Jt, om, oj, os_))
+    out["smc_route_4096x(16+64)"] = dict(ms=ms, flops=2.0 * n_emb * (Md + J) * dim,
+                                         note="latency-bound: 80 dependent 768-dim dots per warp")
+    bank_states = qbank[:n_emb].view(n_emb, -1)
+    sem = torch.zeros((J, bank_states.shape[1]), dtype=torch.float32, device=dev)
+    slots = torch.arange(n_emb, dtype=torch.int64, device=dev) % J
+    ms = timed(lambda: pg.precog_smc_consolidate(sem, bank_states, slots, 0.1), 3)
+    out["smc_consolidate_4096_into_64"] = hbm_row(ms, bank_states.numel() * 2 + 2 * sem.numel() * 4)
+    del sem, flush
+    return out
+
+
 # ------------------------------------------------------------------------------ our arm
 
 
@@ -405,6 +502,11 @@ def main():
                 del b
         del flush
 
+    extras = None
+    if not args.no_extras:
+        extras = measure_extensions(pg, synth, torch, dev, sets[0], off, T, shape.n_chunks, index, qbank,
+                                    query_batch, peaks()[0])
+
     # ---------------- end to end: host inputs -> device -> encode/query -> host results
     e2e = None
     if not args.no_e2e:
@@ -503,7 +605,8 @@ def main():
                            "l2": "inputs larger than L2 (12.98 GB per layer, 1.5 GB index)"},
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks,
                 "gpu_launches": int(launches), "latency": latency,
-                "retrieved_planted": ok_rows, "input_gen_s_per_layer": gen_s_per_layer}
+                "retrieved_planted": ok_rows, "input_gen_s_per_layer": gen_s_per_layer,
+                "extensions": extras}
         print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()

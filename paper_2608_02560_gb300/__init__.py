@@ -227,6 +227,10 @@ def precog_prefill_from_state(inputs: ScanInputs, n_queries: int, T_q: int, bank
         _stream(stream)))
 
 
+def precog_retrieve_topk_workspace_size(M: int, dim: int, n_queries: int) -> int:
+    return int(load_library().precog_retrieve_topk_workspace_size(M, dim, n_queries))
+
+
 def precog_retrieve_topk(index, queries, k, best_idx, best_score=None, workspace=None, stream=None):
     """The k best rows per query into ``best_idx [Q, k]`` (int64) and ``best_score [Q, k]``."""
     import torch

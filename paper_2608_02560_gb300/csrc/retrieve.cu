@@ -152,16 +152,31 @@ __global__ void __launch_bounds__(kThreads)
         partial[static_cast<int64_t>(blockIdx.x) * n_queries + q0 + threadIdx.x] = best[threadIdx.x];
 }
 
+__device__ __forceinline__ unsigned long long shfl_xor_u64(unsigned long long v, int o) {
+    const uint32_t lo = __shfl_xor_sync(0xffffffffu, static_cast<uint32_t>(v), o);
+    const uint32_t hi = __shfl_xor_sync(0xffffffffu, static_cast<uint32_t>(v >> 32), o);
+    return (static_cast<unsigned long long>(hi) << 32) | lo;
+}
+
+// One warp per query: each lane takes the maximum over a strided share of the
+// per-CTA keys (independent loads, so many are in flight), then a butterfly.
 __global__ void finalize_kernel(const unsigned long long *__restrict__ partial, int n_parts,
                                 int n_queries, int64_t *__restrict__ best_idx,
                                 float *__restrict__ best_score) {
-    const int q = blockIdx.x * blockDim.x + threadIdx.x;
+    const int q = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
     if (q >= n_queries) return;
     unsigned long long k = 0ull;
-    for (int i = 0; i < n_parts; ++i) {
+    for (int i = lane; i < n_parts; i += 32) {
         const unsigned long long v = partial[static_cast<int64_t>(i) * n_queries + q];
         k = v > k ? v : k;
     }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const unsigned long long v = shfl_xor_u64(k, o);
+        k = v > k ? v : k;
+    }
+    if (lane != 0) return;
     if (k == 0ull) {
         best_idx[q] = -1;
         if (best_score) best_score[q] = __uint_as_float(0x7fc00000u);
@@ -242,7 +257,12 @@ __global__ void __launch_bounds__(kThreads)
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
             const int64_t row = r0 + r;
-            if (row < M && !isnan(acc)) list_insert(l, make_key(acc, row));
+            // acc is the same in every lane (xor butterfly), so the branch is uniform;
+            // most rows fall below the list's last key and skip the insertion
+            if (row < M && !isnan(acc)) {
+                const unsigned long long key = make_key(acc, row);
+                if (key > l[kListK - 1]) list_insert(l, key);
+            }
         }
     }
     if (lane == 0)
@@ -262,21 +282,34 @@ __global__ void __launch_bounds__(kThreads)
     }
 }
 
-// Merge the per-CTA lists of one query (one thread per query) into its k best.
+// Merge the per-CTA lists of one query into its k best, one warp per query:
+// each lane merges a strided share of the CTAs' lists, then five butterfly
+// rounds merge the lanes' lists (keys are unique, so both partners of a round
+// end with the same list).
 __global__ void finalize_topk_kernel(const unsigned long long *__restrict__ partial, int n_parts,
                                      int n_queries, int k, int64_t *__restrict__ best_idx,
                                      float *__restrict__ best_score) {
-    const int q = blockIdx.x * blockDim.x + threadIdx.x;
+    const int q = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
     if (q >= n_queries) return;
     unsigned long long l[kListK];
 #pragma unroll
     for (int j = 0; j < kListK; ++j) l[j] = 0ull;
-    for (int i = 0; i < n_parts; ++i)
+    for (int i = lane; i < n_parts; i += 32)
         for (int j = 0; j < kListK; ++j) {
             const unsigned long long v = partial[(static_cast<int64_t>(i) * n_queries + q) * kListK + j];
             if (v <= l[kListK - 1]) break;   // each part's list is sorted: the rest is smaller
             list_insert(l, v);
         }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        unsigned long long other[kListK];
+#pragma unroll
+        for (int j = 0; j < kListK; ++j) other[j] = shfl_xor_u64(l[j], o);
+#pragma unroll
+        for (int j = 0; j < kListK; ++j) list_insert(l, other[j]);
+    }
+    if (lane != 0) return;
     for (int j = 0; j < k; ++j) {
         const unsigned long long key = l[j];
         const int64_t o = static_cast<int64_t>(q) * k + j;
@@ -403,7 +436,7 @@ cudaError_t launch_retrieve(const RetrieveParams &p, cudaStream_t stream) {
         }
     }
     if (e == cudaSuccess) {
-        finalize_kernel<<<(p.n_queries + 127) / 128, 128, 0, stream>>>(
+        finalize_kernel<<<(p.n_queries + 3) / 4, 128, 0, stream>>>(
             static_cast<const unsigned long long *>(p.workspace), parts, p.n_queries, p.best_idx,
             p.best_score);
         e = cudaGetLastError();
@@ -439,7 +472,7 @@ cudaError_t launch_retrieve_topk(const RetrieveParams &p, int k, cudaStream_t st
         }
     }
     if (e == cudaSuccess) {
-        finalize_topk_kernel<<<(p.n_queries + 127) / 128, 128, 0, stream>>>(
+        finalize_topk_kernel<<<(p.n_queries + 3) / 4, 128, 0, stream>>>(
             static_cast<const unsigned long long *>(p.workspace), parts, p.n_queries, k, p.best_idx,
             p.best_score);
         e = cudaGetLastError();

@@ -233,31 +233,38 @@ __global__ void __launch_bounds__(kThreads, 1)
                                   static_cast<uint32_t>(acc * 2 * kBN + h * kBN + c0),
                               v);
                     const int64_t rbase = row0 + c0;
-                    if constexpr (LIST == 1) {
-                        if (rbase + 32 <= M) {
+                    // Fast path: the column maximum of the 32 values (NaN ignored). Only
+                    // when it beats the running best (rare after the first tiles) are the
+                    // columns scanned again in increasing order with a strict '>', so the
+                    // lowest row still wins ties.
+                    const bool full_cols = rbase + 32 <= M;
+                    float m = -__int_as_float(0x7f800000);
+                    if (full_cols) {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) m = fmaxf(m, v[j]);
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            if (rbase + j < M) m = fmaxf(m, v[j]);
+                    }
+                    if (m > best[h]) {
+                        if constexpr (LIST == 1) {
 #pragma unroll
                             for (int j = 0; j < 32; ++j)
-                                if (v[j] > best[h]) {
+                                if ((full_cols || rbase + j < M) && v[j] > best[h]) {
                                     best[h] = v[j];
                                     best_row[h] = rbase + j;
                                 }
                         } else {
+                            // best[h] tracks the list's last score
 #pragma unroll
                             for (int j = 0; j < 32; ++j)
-                                if (rbase + j < M && v[j] > best[h]) {
-                                    best[h] = v[j];
-                                    best_row[h] = rbase + j;
+                                if ((full_cols || rbase + j < M) && v[j] > best[h]) {
+                                    tc_list_insert<LIST>(lst[h], tc_key(v[j], rbase + j));
+                                    if (lst[h][LIST - 1] != 0ull)
+                                        best[h] = unordered_tc(static_cast<uint32_t>(lst[h][LIST - 1] >> 32));
                                 }
                         }
-                    } else {
-                        // best[h] tracks the list's last score: one compare per column
-#pragma unroll
-                        for (int j = 0; j < 32; ++j)
-                            if (rbase + j < M && v[j] > best[h]) {
-                                tc_list_insert<LIST>(lst[h], tc_key(v[j], rbase + j));
-                                if (lst[h][LIST - 1] != 0ull)
-                                    best[h] = unordered_tc(static_cast<uint32_t>(lst[h][LIST - 1] >> 32));
-                            }
                     }
                 }
             }

@@ -70,16 +70,19 @@ __device__ __forceinline__ int64_t min64(int64_t a, int64_t b) { return a < b ? 
 enum Mode { kGeneral = 0, kPower = 1 };
 
 // Compile-time shape of one kernel instantiation.
+constexpr int kTrajNone = 0, kTrajDirect = 1, kTrajRescaled = 2;
+
 template <typename TIn_, bool HAS_Y_, bool HAS_H0_, int MODE_, int CPT_, int TILE_, int STAGES_,
-          int MINB_, bool TRAJ_ = false>
+          int MINB_, int TRAJ_ = kTrajNone>
 struct Cfg {
     using TIn = TIn_;
     static constexpr bool HAS_Y = HAS_Y_, HAS_H0 = HAS_H0_;
-    static constexpr bool TRAJ = TRAJ_;     // keep every stride-th state (K-dial, Sec. 5.2)
+    // keep every stride-th state (K-dial, Sec. 5.2), with the direct or the rescaled update
+    static constexpr int TRAJ = TRAJ_;
     static constexpr int MODE = MODE_, CPT = CPT_, TILE = TILE_, STAGES = STAGES_, MINB = MINB_;
     static constexpr bool CONV = !std::is_same<TIn_, float>::value;
     static constexpr int SZ = sizeof(TIn_);
-    static constexpr bool RESCALED = MODE_ == kPower && !HAS_Y_ && !TRAJ_;
+    static constexpr bool RESCALED = MODE_ == kPower && !HAS_Y_ && TRAJ_ != kTrajDirect;
 };
 
 // Where the next trajectory state goes: entry index and tokens left until it.
@@ -298,7 +301,7 @@ __device__ __forceinline__ void scan_tile_direct(const unsigned char *st, const 
                 }
             }
         }
-        if constexpr (C::TRAJ) {
+        if constexpr (C::TRAJ == kTrajDirect) {
             // after every stride-th token and after the chunk's last token (uniform)
             if (--tc.left == 0 || t + 1 == tok_left) {
 #pragma unroll
@@ -397,13 +400,13 @@ constexpr int kGroup = PRECOG_RESCALED_GROUP;
 
 template <class C>
 __device__ __forceinline__ void scan_tile_rescaled(const unsigned char *st, const StageLayout &lay,
-                                                   int DS, int dl, int ntok,
+                                                   int DS, int dl, int t0, int ntok,
                                                    f2 (&g)[C::CPT][8], float (&L)[C::CPT],
                                                    const float (&kk)[C::CPT], unsigned wmask) {
     constexpr int CPT = C::CPT;
     using TIn = typename C::TIn;
     const float *bsrc = reinterpret_cast<const float *>(st + (C::CONV ? lay.bf : lay.bs));
-    int t = 0;
+    int t = t0;
     for (; t + kGroup <= ntok; t += kGroup) {
         float dvk[kGroup][CPT], Lk[kGroup][CPT];
         uint32_t neg = 0;
@@ -675,8 +678,30 @@ __global__ void __launch_bounds__(kMaxSlice / C::CPT, C::MINB)
             }
             return;
         }
-        if constexpr (C::RESCALED) {
-            scan_tile_rescaled<C>(st, lay, DS, dl, ntok, h, Lw, kk, wmask);
+        if constexpr (C::RESCALED && C::TRAJ == kTrajRescaled) {
+            // segments end at the trajectory points; there the state is brought back
+            // to h (renormalised, L = 0), stored, and the accumulation continues
+            int t = 0;
+            while (t < ntok) {
+                const int seg = static_cast<int>(min64(ntok - t, tcur.left));
+                scan_tile_rescaled<C>(st, lay, DS, dl, t, t + seg, h, Lw, kk, wmask);
+                t += seg;
+                tcur.left -= seg;
+                if (tcur.left == 0 || k * TILE + t == len) {
+#pragma unroll
+                    for (int j = 0; j < CPT; ++j) {
+                        renormalise(h[j], Lw[j]);
+                        store_state16(p.traj, p.traj_dtype,
+                                      ((tcur.entry * p.L_out + p.layer0 + layer) * static_cast<int64_t>(D) +
+                                       d0 + dl + j) * kN,
+                                      h[j]);
+                    }
+                    ++tcur.entry;
+                    tcur.left = p.traj_stride;
+                }
+            }
+        } else if constexpr (C::RESCALED) {
+            scan_tile_rescaled<C>(st, lay, DS, dl, 0, ntok, h, Lw, kk, wmask);
         } else {
             scan_tile_direct<C>(st, lay, DS, dl, ntok, h, kpow, kgen, yrow, p.y_dtype, y_stride, p, tcur,
                                 len - k * TILE, p.layer0 + layer, d0 + dl);
@@ -737,15 +762,18 @@ cudaError_t launch_cfg(const ScanParams &p, cudaStream_t stream) {
 
 // Shapes: the rescaled capture kernel (the corpus-encode hot loop) and the
 // direct kernels (readout, prefill, general A).
-template <typename TIn, bool HAS_Y, bool HAS_H0, int MODE, bool TRAJ = false>
+template <typename TIn, bool HAS_Y, bool HAS_H0, int MODE, int TRAJ = kTrajNone>
 cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
-    if constexpr (TRAJ) {
-        // trajectory capture uses the direct update (the state is needed every stride tokens)
+    if constexpr (TRAJ == kTrajRescaled) {
+        return launch_cfg<Cfg<TIn, false, false, kPower, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
+                              PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB, kTrajRescaled>>(p, stream);
+    } else if constexpr (TRAJ == kTrajDirect) {
+        // short strides and general A: the direct update (h is at hand after every token)
         if constexpr (MODE == kPower)
             return launch_cfg<Cfg<TIn, false, false, MODE, PRECOG_DIRECT_CPT, PRECOG_DIRECT_TILE,
-                                  PRECOG_DIRECT_STAGES, PRECOG_DIRECT_MINB, true>>(p, stream);
+                                  PRECOG_DIRECT_STAGES, PRECOG_DIRECT_MINB, kTrajDirect>>(p, stream);
         else
-            return launch_cfg<Cfg<TIn, false, false, MODE, 2, 16, 4, 3, true>>(p, stream);
+            return launch_cfg<Cfg<TIn, false, false, MODE, 2, 16, 4, 3, kTrajDirect>>(p, stream);
     } else if constexpr (MODE == kPower && !HAS_Y) {
         return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
                               PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB>>(p, stream);
@@ -762,7 +790,13 @@ cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
 
 template <typename TIn, int MODE>
 cudaError_t launch_mode(const ScanParams &p, cudaStream_t stream) {
-    if (p.traj != nullptr) return launch_t<TIn, false, false, MODE, true>(p, stream);
+    if (p.traj != nullptr) {
+        // strides of at least a few token groups amortise the renormalisation at each
+        // trajectory point, so they take the rescaled accumulation
+        if constexpr (MODE == kPower)
+            if (p.traj_stride >= 4 * kGroup) return launch_t<TIn, false, false, MODE, kTrajRescaled>(p, stream);
+        return launch_t<TIn, false, false, MODE, kTrajDirect>(p, stream);
+    }
     const bool has_y = p.y != nullptr;
     const bool has_h0 = p.bank != nullptr;
     if (has_y)

@@ -40,6 +40,35 @@ __device__ __forceinline__ float ld(const TIn *p) {
     return to_f32(__ldg(p));
 }
 
+// One 16-value B or C row (32 or 64 bytes, 16-byte aligned) with vector loads;
+// every thread of the block reads the same row, so a warp issues one request.
+template <typename TIn>
+__device__ __forceinline__ void ld_row16(const TIn *row, float (&v)[kN]) {
+    if constexpr (std::is_same<TIn, float>::value) {
+        const float4 *r = reinterpret_cast<const float4 *>(row);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float4 q = __ldg(r + i);
+            v[4 * i] = q.x;
+            v[4 * i + 1] = q.y;
+            v[4 * i + 2] = q.z;
+            v[4 * i + 3] = q.w;
+        }
+    } else {
+        const uint4 *r = reinterpret_cast<const uint4 *>(row);
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+            const uint4 q = __ldg(r + i);
+            const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                v[8 * i + 2 * k] = __uint_as_float(w[k] << 16);
+                v[8 * i + 2 * k + 1] = __uint_as_float(w[k] & 0xffff0000u);
+            }
+        }
+    }
+}
+
 template <typename TIn, bool HAS_Y, bool HAS_H0>
 __global__ void __launch_bounds__(kBlock)
     scan_complex_kernel(const ScanParams p, const int cblocks) {
@@ -103,6 +132,9 @@ __global__ void __launch_bounds__(kBlock)
         const float xv = ld(xl + t * D + d);
         const float dv = ld(dtl + t * D + d);
         const float u = dv * xv;
+        float b[kN], cr[kN];
+        ld_row16<TIn>(Bl + t * kN, b);
+        if constexpr (HAS_Y) ld_row16<TIn>(Cl + t * kN, cr);
         float y = 0.f;
 #pragma unroll
         for (int n = 0; n < kN; ++n) {
@@ -112,11 +144,11 @@ __global__ void __launch_bounds__(kBlock)
             float s, c;
             sincos_reduced(th, tl, s, c);
             const float are = mag * c, aim = mag * s;
-            const float nr = fmaf(are, hr[n], fmaf(-aim, hi[n], u * ld(Bl + t * kN + n)));
+            const float nr = fmaf(are, hr[n], fmaf(-aim, hi[n], u * b[n]));
             const float ni = fmaf(are, hi[n], aim * hr[n]);
             hr[n] = nr;
             hi[n] = ni;
-            if constexpr (HAS_Y) y = fmaf(ld(Cl + t * kN + n), nr, y);
+            if constexpr (HAS_Y) y = fmaf(cr[n], nr, y);
         }
         if constexpr (HAS_Y) {
             const int64_t yo = (static_cast<int64_t>(layer) * p.T_tot + t) * D + d;

@@ -72,24 +72,86 @@ __global__ void __launch_bounds__(kRouteWarps * 32)
 }
 
 // s[slot_c] <- (1 - alpha) s[slot_c] + alpha h_c for c = 0, 1, ... in order,
-// one thread per state element; slot -1 deposits nothing.
+// one thread per state element. Deposits go in batches of kU: the batch's
+// slots are read once into shared memory (uniform across the block), every
+// thread issues the batch's state loads and slot loads together, folds the
+// batch in deposit order and stores each touched slot once. When a slot
+// repeats inside a batch the fold runs through a per-thread shared-memory
+// column so that each repeat starts from the value its predecessor left.
+// Slot -1 deposits nothing; a slot >= n_slots is flagged and skipped.
+constexpr int kU = 32;
+constexpr int kConsThreads = 256;
+
 template <typename TS>
-__global__ void smc_consolidate_kernel(float *__restrict__ sem, int64_t n_slots, int64_t elems,
-                                       const TS *__restrict__ states, const int64_t *__restrict__ slots,
-                                       int64_t n, float alpha) {
+__global__ void __launch_bounds__(kConsThreads, 2)
+    smc_consolidate_kernel(float *__restrict__ sem, int64_t n_slots, int64_t elems,
+                           const TS *__restrict__ states, const int64_t *__restrict__ slots,
+                           int64_t n, float alpha) {
+    __shared__ int64_t s_slot[kU];
+    __shared__ int64_t s_off[kU];   // slot * elems
+    __shared__ int s_prev[kU];      // latest earlier position of the same slot in the batch, or -1
+    __shared__ int s_last[kU];      // no later position of the batch has the same slot
+    __shared__ int s_dups;
+    __shared__ float s_val[kU][kConsThreads];
     const float keep = 1.f - alpha;
-    for (int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < elems;
-         e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        for (int64_t c = 0; c < n; ++c) {
-            const int64_t slot = slots[c];
-            if (slot < 0) continue;
-            if (slot >= n_slots) {
-                if (e == 0) atomicOr(&g_smc_status, PRECOG_DEV_BAD_INDEX);
-                continue;
+    const int tid = threadIdx.x;
+    const int64_t e = static_cast<int64_t>(blockIdx.x) * kConsThreads + tid;
+    for (int64_t c0 = 0; c0 < n; c0 += kU) {
+        __syncthreads();                       // the previous batch is done with s_*
+        if (tid < kU) {
+            const int64_t c = c0 + tid;
+            int64_t sl = c < n ? slots[c] : -1;
+            if (sl >= n_slots) {
+                if (blockIdx.x == 0) atomicOr(&g_smc_status, PRECOG_DEV_BAD_INDEX);
+                sl = -1;
             }
-            float *s = sem + slot * elems + e;
-            *s = keep * *s + alpha * to_f32(states[c * elems + e]);
+            if (sl < -1) sl = -1;
+            s_slot[tid] = sl;
+            s_off[tid] = sl >= 0 ? sl * elems : 0;
         }
+        if (tid == 0) s_dups = 0;
+        __syncthreads();
+        if (tid < kU) {
+            const int64_t sl = s_slot[tid];
+            int prev = -1, last = 1;
+            if (sl >= 0) {
+                for (int i = 0; i < tid; ++i)
+                    if (s_slot[i] == sl) prev = i;
+                for (int i = tid + 1; i < kU; ++i)
+                    if (s_slot[i] == sl) last = 0;
+            }
+            s_prev[tid] = prev;
+            s_last[tid] = last;
+            if (prev >= 0) atomicOr(&s_dups, 1);
+        }
+        __syncthreads();
+        if (e >= elems) continue;
+        float h[kU], v[kU];
+#pragma unroll
+        for (int j = 0; j < kU; ++j) {
+            h[j] = 0.f;
+            v[j] = 0.f;
+            if (s_slot[j] >= 0) h[j] = to_f32(states[(c0 + j) * elems + e]);
+        }
+#pragma unroll
+        for (int j = 0; j < kU; ++j)
+            if (s_slot[j] >= 0 && s_prev[j] < 0) v[j] = sem[s_off[j] + e];
+        if (!s_dups) {
+#pragma unroll
+            for (int j = 0; j < kU; ++j) v[j] = fmaf(keep, v[j], alpha * h[j]);
+        } else {
+#pragma unroll
+            for (int j = 0; j < kU; ++j) {
+                if (s_slot[j] < 0) continue;
+                const int pj = s_prev[j];
+                const float base = pj >= 0 ? s_val[pj][tid] : v[j];
+                v[j] = fmaf(keep, base, alpha * h[j]);
+                s_val[j][tid] = v[j];
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < kU; ++j)
+            if (s_slot[j] >= 0 && s_last[j]) sem[s_off[j] + e] = v[j];
     }
 }
 
@@ -136,14 +198,14 @@ cudaError_t launch_smc_consolidate(float *sem, int64_t n_slots, int64_t elems, c
                                    int states_dtype, const int64_t *slots, int64_t n, float alpha,
                                    cudaStream_t stream) {
     if (n == 0 || elems == 0) return cudaSuccess;
-    const int threads = 256;
-    const int64_t want = (elems + threads - 1) / threads;
-    const unsigned grid = static_cast<unsigned>(want < sm_count() * 16 ? want : sm_count() * 16);
+    const int64_t blocks = (elems + kConsThreads - 1) / kConsThreads;
+    if (blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+    const unsigned grid = static_cast<unsigned>(blocks);
     if (states_dtype == PRECOG_BF16)
-        smc_consolidate_kernel<__nv_bfloat16><<<grid, threads, 0, stream>>>(
+        smc_consolidate_kernel<__nv_bfloat16><<<grid, kConsThreads, 0, stream>>>(
             sem, n_slots, elems, static_cast<const __nv_bfloat16 *>(states), slots, n, alpha);
     else
-        smc_consolidate_kernel<float><<<grid, threads, 0, stream>>>(
+        smc_consolidate_kernel<float><<<grid, kConsThreads, 0, stream>>>(
             sem, n_slots, elems, static_cast<const float *>(states), slots, n, alpha);
     cudaError_t e = cudaGetLastError();
     if (e == cudaSuccess) count_launches(1);

@@ -72,3 +72,51 @@ def test_consolidate_then_session_init(cuda_device):
             ref_h, _ = oracle.rollout(to_np(x[l, sl]), to_np(dt[l, sl]), An, to_np(B[l, sl]),
                                       h0=ref[srow].reshape(L, D, N)[l])
             assert rel_err(to_np(h[q, l]), ref_h) < TOL_F32
+
+
+@pytest.mark.parametrize("n,n_slots,pattern", [(200, 64, "cyclic"), (77, 3, "runs"), (1, 5, "cyclic"),
+                                               (96, 40, "random")])
+def test_consolidate_deposit_patterns(cuda_device, n, n_slots, pattern):
+    """Deposit orders that exercise the batched fold: no slot repeated within a batch
+    (cyclic), long runs of one slot, a single deposit, random slots with -1 mixed in;
+    fp32 states of an odd element count."""
+    import torch
+    import paper_2608_02560_gb300 as pg
+    rng = np.random.default_rng(n + n_slots)
+    elems = 333
+    states = rng.standard_normal((n, elems)).astype(np.float32)
+    if pattern == "cyclic":
+        slot_np = np.arange(n, dtype=np.int64) % n_slots
+    elif pattern == "runs":
+        slot_np = (np.arange(n, dtype=np.int64) // 10) % n_slots
+    else:
+        slot_np = rng.integers(-1, n_slots, size=n).astype(np.int64)
+    sem0 = rng.standard_normal((n_slots, elems)).astype(np.float32)
+    sem = torch.from_numpy(sem0).to(cuda_device)
+    pg.precog_smc_consolidate(sem, torch.from_numpy(states).to(cuda_device),
+                              torch.from_numpy(slot_np).to(cuda_device), 0.3)
+    assert pg.precog_device_status()[0] == 0
+    ref = oracle.smc_consolidate(sem0, states, slot_np, 0.3)
+    got = to_np(sem)
+    for s in range(n_slots):
+        assert rel_err(got[s], ref[s]) < TOL_F32, s
+
+
+def test_consolidate_flags_slot_outside_table(cuda_device):
+    """A slot >= n_slots deposits nothing and raises PRECOG_DEV_BAD_INDEX; the other
+    deposits still apply."""
+    import torch
+    import paper_2608_02560_gb300 as pg
+    rng = np.random.default_rng(5)
+    states = rng.standard_normal((6, 64)).astype(np.float32)
+    slot_np = np.array([0, 1, 9, 1, 0, 2], dtype=np.int64)      # 9 is outside a 3-slot table
+    sem0 = np.zeros((3, 64), dtype=np.float32)
+    sem = torch.from_numpy(sem0).to(cuda_device)
+    pg.precog_smc_consolidate(sem, torch.from_numpy(states).to(cuda_device),
+                              torch.from_numpy(slot_np).to(cuda_device), 0.5)
+    st, bits = pg.precog_device_status()
+    assert st != 0 and bits & pg.PRECOG_DEV_BAD_INDEX
+    keep = slot_np.copy()
+    keep[2] = -1
+    ref = oracle.smc_consolidate(sem0, states, keep, 0.5)
+    assert rel_err(to_np(sem), ref) < TOL_F32

@@ -23,7 +23,7 @@ def _run(dev, x, dt, B, A, off, stride, dtype, power, layer0=0, L_total=1):
     return traj
 
 
-@pytest.mark.parametrize("stride", [1, 5, 16, 64, 1000])
+@pytest.mark.parametrize("stride", [1, 5, 16, 17, 64, 1000])
 @pytest.mark.parametrize("power", [False, True])
 def test_trajectory_fp32(cuda_device, stride, power):
     """Ragged chunks (incl. empty and single-token), fp32: every kept state vs the oracle."""
