@@ -61,7 +61,7 @@ def parse_args():
     ap.add_argument("--no-latency", action="store_true")
     ap.add_argument("--no-extras", action="store_true",
                     help="skip the measurements of the extension rows (top-k, trajectory, complex A, SMC)")
-    ap.add_argument("--case", choices=["full", "scan-small", "retrieve-small", "prefill-small"],
+    ap.add_argument("--case", choices=["full", "scan-small", "retrieve-small", "topk-small", "prefill-small"],
                     default="full",
                     help="small single-kernel cases (a few GB) used for profiler captures")
     return ap.parse_args()
@@ -220,12 +220,17 @@ def run_case(args):
         fn = lambda: pg.precog_encode_chunks(si, off, T, states_out=bank, layer0=0, L_total=shape.n_layers)
         res["algorithmic_bytes_per_launch"] = scan_bytes_per_launch(T, chunks, shape.D, shape.N)
         res["scale_to_full_launch"] = shape.n_chunks * shape.chunk_len / T
-    elif args.case == "retrieve-small":
+    elif args.case in ("retrieve-small", "topk-small"):
         M = 1 << 18
         index = synth.device_unit_index(M, synth.QUERY_DIM, 0, dev)
         q, _ = synth.device_planted_queries(index, args.query_batch, synth.QUERY_NOISE, 1)
-        idx = torch.empty(args.query_batch, dtype=torch.int64, device=dev)
-        fn = lambda: pg.precog_retrieve(index, q, idx)
+        if args.case == "retrieve-small":
+            idx = torch.empty(args.query_batch, dtype=torch.int64, device=dev)
+            fn = lambda: pg.precog_retrieve(index, q, idx)
+        else:
+            idx = torch.empty((args.query_batch, 3), dtype=torch.int64, device=dev)
+            sc = torch.empty((args.query_batch, 3), dtype=torch.float32, device=dev)
+            fn = lambda: pg.precog_retrieve_topk(index, q, 3, idx, sc)
         res["algorithmic_bytes_per_launch"] = M * synth.QUERY_DIM * 2
     else:
         L, D, N, Tq, Q, entries = 24, 256, 16, synth.QUERY_TOKENS, args.query_batch, 4096

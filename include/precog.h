@@ -313,6 +313,9 @@ precog_status precog_smc_route(const void *embeddings, int32_t dtype, int64_t n,
  *                chunks' K = 1 states from precog_encode_chunks
  *   d_slots      device int64 [n], e.g. precog_smc_route's d_slot
  *   alpha        in (0, 1]
+ * semantic and states must be 16-byte aligned (else PRECOG_ERR_INVALID_ARG).
+ * Each element's deposits are applied in deposit order, so the result does not
+ * depend on how the work is split.
  */
 precog_status precog_smc_consolidate(float *semantic, int64_t n_slots, int64_t state_elems,
                                      const void *states, int32_t states_dtype, const int64_t *d_slots,

@@ -405,6 +405,8 @@ precog_status precog_smc_consolidate(float *semantic, int64_t n_slots, int64_t s
     if (n == 0 || state_elems == 0) return ok();
     if (semantic == nullptr || states == nullptr || d_slots == nullptr)
         return fail(PRECOG_ERR_INVALID_ARG, "semantic, states and d_slots must be non-NULL");
+    if (!aligned16(semantic) || !aligned16(states))
+        return fail(PRECOG_ERR_INVALID_ARG, "semantic and states must be 16-byte aligned");
     cudaError_t e = precog::launch_smc_consolidate(semantic, n_slots, state_elems, states, states_dtype,
                                                    d_slots, n, alpha, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "smc consolidate launch");

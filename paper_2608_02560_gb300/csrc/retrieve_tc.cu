@@ -48,6 +48,8 @@ struct Smem {
     uint64_t acc_empty[2];
     uint32_t tmem_base;
     uint32_t abort_flag;
+    // epilogue scratch: one row of 32 scores per epilogue thread (padded: conflict-free)
+    float epi[4 * 32][33];
 };
 
 // Shared-memory matrix descriptor: K-major operand, 128B swizzle, rows of 128
@@ -208,6 +210,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---------------- epilogue: argmax over key rows, per query ----------------
         const int quarter = warp & 3;                 // TMEM lanes 32*quarter .. +31
         const int qrow = quarter * 32 + lane;         // query row inside a half
+        const int ethr = threadIdx.x - 64;            // scratch row of this epilogue thread
         float best[2] = {-__int_as_float(0x7f800000), -__int_as_float(0x7f800000)};
         int64_t best_row[2] = {-1, -1};
         unsigned long long lst[2][LIST > 1 ? LIST : 1];
@@ -248,22 +251,32 @@ __global__ void __launch_bounds__(kThreads, 1)
                             if (rbase + j < M) m = fmaxf(m, v[j]);
                     }
                     if (m > best[h]) {
-                        if constexpr (LIST == 1) {
+                        // Slow path (rare per thread, but a warp takes it whenever one of
+                        // its 32 queries does): mark the columns that beat the running
+                        // best, park the scores in this thread's scratch row and visit
+                        // only the marked ones, lowest column first. A compact loop keeps
+                        // the epilogue's code small.
+                        uint32_t mask = 0u;
 #pragma unroll
-                            for (int j = 0; j < 32; ++j)
-                                if ((full_cols || rbase + j < M) && v[j] > best[h]) {
-                                    best[h] = v[j];
-                                    best_row[h] = rbase + j;
-                                }
-                        } else {
-                            // best[h] tracks the list's last score
-#pragma unroll
-                            for (int j = 0; j < 32; ++j)
-                                if ((full_cols || rbase + j < M) && v[j] > best[h]) {
-                                    tc_list_insert<LIST>(lst[h], tc_key(v[j], rbase + j));
-                                    if (lst[h][LIST - 1] != 0ull)
-                                        best[h] = unordered_tc(static_cast<uint32_t>(lst[h][LIST - 1] >> 32));
-                                }
+                        for (int j = 0; j < 32; ++j) {
+                            const bool in = (full_cols || rbase + j < M) && v[j] > best[h];
+                            mask |= in ? (1u << j) : 0u;
+                            sm.epi[ethr][j] = v[j];
+                        }
+                        while (mask) {
+                            const int j = __ffs(static_cast<int>(mask)) - 1;
+                            mask &= mask - 1u;
+                            const float val = sm.epi[ethr][j];
+                            if (!(val > best[h])) continue;
+                            if constexpr (LIST == 1) {
+                                best[h] = val;
+                                best_row[h] = rbase + j;
+                            } else {
+                                // best[h] tracks the list's last score
+                                tc_list_insert<LIST>(lst[h], tc_key(val, rbase + j));
+                                if (lst[h][LIST - 1] != 0ull)
+                                    best[h] = unordered_tc(static_cast<uint32_t>(lst[h][LIST - 1] >> 32));
+                            }
                         }
                     }
                 }

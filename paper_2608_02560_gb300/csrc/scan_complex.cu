@@ -35,39 +35,34 @@ __device__ __forceinline__ void sincos_reduced(float hi, float lo, float &s, flo
     asm("cos.approx.ftz.f32 %0, %1;" : "=f"(c) : "f"(r));
 }
 
+// One 16-value B or C row (32 or 64 bytes, 16-byte aligned), fetched raw with
+// vector loads one token ahead of its use; every thread of the block reads the
+// same row, so a warp issues one request per vector.
 template <typename TIn>
-__device__ __forceinline__ float ld(const TIn *p) {
-    return to_f32(__ldg(p));
-}
-
-// One 16-value B or C row (32 or 64 bytes, 16-byte aligned) with vector loads;
-// every thread of the block reads the same row, so a warp issues one request.
-template <typename TIn>
-__device__ __forceinline__ void ld_row16(const TIn *row, float (&v)[kN]) {
-    if constexpr (std::is_same<TIn, float>::value) {
-        const float4 *r = reinterpret_cast<const float4 *>(row);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const float4 q = __ldg(r + i);
-            v[4 * i] = q.x;
-            v[4 * i + 1] = q.y;
-            v[4 * i + 2] = q.z;
-            v[4 * i + 3] = q.w;
-        }
-    } else {
+struct RawRow {
+    static constexpr int kVec = static_cast<int>(kN * sizeof(TIn) / 16);
+    uint4 q[kVec];
+    __device__ __forceinline__ void load(const TIn *row) {
         const uint4 *r = reinterpret_cast<const uint4 *>(row);
 #pragma unroll
-        for (int i = 0; i < 2; ++i) {
-            const uint4 q = __ldg(r + i);
-            const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+        for (int i = 0; i < kVec; ++i) q[i] = __ldg(r + i);
+    }
+    __device__ __forceinline__ void widen(float (&v)[kN]) const {
+#pragma unroll
+        for (int i = 0; i < kVec; ++i) {
+            const uint32_t w[4] = {q[i].x, q[i].y, q[i].z, q[i].w};
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
-                v[8 * i + 2 * k] = __uint_as_float(w[k] << 16);
-                v[8 * i + 2 * k + 1] = __uint_as_float(w[k] & 0xffff0000u);
+                if constexpr (std::is_same<TIn, float>::value) {
+                    v[4 * i + k] = __uint_as_float(w[k]);
+                } else {
+                    v[8 * i + 2 * k] = __uint_as_float(w[k] << 16);
+                    v[8 * i + 2 * k + 1] = __uint_as_float(w[k] & 0xffff0000u);
+                }
             }
         }
     }
-}
+};
 
 template <typename TIn, bool HAS_Y, bool HAS_H0>
 __global__ void __launch_bounds__(kBlock)
@@ -128,13 +123,29 @@ __global__ void __launch_bounds__(kBlock)
             atomicOr(&g_scan_complex_status, PRECOG_DEV_BAD_INDEX);
         }
     }
-    for (int64_t t = start; t < start + len; ++t) {
-        const float xv = ld(xl + t * D + d);
-        const float dv = ld(dtl + t * D + d);
+    // token t+1's inputs are in flight while token t is computed
+    TIn nx{}, ndt{};
+    RawRow<TIn> nb{}, nc{};
+    const int64_t end = start + len;
+    if (len > 0) {
+        nx = xl[start * D + d];
+        ndt = dtl[start * D + d];
+        nb.load(Bl + start * kN);
+        if constexpr (HAS_Y) nc.load(Cl + start * kN);
+    }
+    for (int64_t t = start; t < end; ++t) {
+        const float xv = to_f32(nx);
+        const float dv = to_f32(ndt);
         const float u = dv * xv;
         float b[kN], cr[kN];
-        ld_row16<TIn>(Bl + t * kN, b);
-        if constexpr (HAS_Y) ld_row16<TIn>(Cl + t * kN, cr);
+        nb.widen(b);
+        if constexpr (HAS_Y) nc.widen(cr);
+        if (t + 1 < end) {
+            nx = xl[(t + 1) * D + d];
+            ndt = dtl[(t + 1) * D + d];
+            nb.load(Bl + (t + 1) * kN);
+            if constexpr (HAS_Y) nc.load(Cl + (t + 1) * kN);
+        }
         float y = 0.f;
 #pragma unroll
         for (int n = 0; n < kN; ++n) {

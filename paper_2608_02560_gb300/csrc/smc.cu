@@ -2,6 +2,8 @@
 // routing (Eqs. smc-domain, smc-sub) and the semantic-state EMA (Eq. smc-ema).
 // Session initialisation (Sec. 5.3) injects a semantic state with the
 // ordinary prefill, so it needs no kernel of its own.
+#include <climits>
+#include <cstdint>
 #include <type_traits>
 
 #include "../../include/precog.h"
@@ -72,98 +74,146 @@ __global__ void __launch_bounds__(kRouteWarps * 32)
 }
 
 // s[slot_c] <- (1 - alpha) s[slot_c] + alpha h_c for c = 0, 1, ... in order,
-// one thread per state element. Deposits go in batches of kU: the batch's
-// slots are read once into shared memory (uniform across the block), every
-// thread issues the batch's state loads and slot loads together, folds the
-// batch in deposit order and stores each touched slot once. When a slot
-// repeats inside a batch the fold runs through a per-thread shared-memory
-// column so that each repeat starts from the value its predecessor left.
+// one thread per VEC adjacent state elements. Deposits go in batches of kU:
+// warp 0 reads a batch's slots and describes it for the whole block (per
+// deposit: the slot's offset, the latest earlier deposit of the same slot in
+// the batch, whether a later one follows), one batch ahead, with a match-any
+// vote instead of pairwise compares. Every thread then issues the batch's
+// state loads and first-touch slot loads together, folds the batch in deposit
+// order (a repeat inside the batch starts from its predecessor's result, kept
+// in a per-thread shared-memory column) and stores each touched slot once.
 // Slot -1 deposits nothing; a slot >= n_slots is flagged and skipped.
-constexpr int kU = 32;
-constexpr int kConsThreads = 256;
+constexpr int kU = 16;
+constexpr int kConsThreads = 128;
 
-template <typename TS>
-__global__ void __launch_bounds__(kConsThreads, 2)
-    smc_consolidate_kernel(float *__restrict__ sem, int64_t n_slots, int64_t elems,
-                           const TS *__restrict__ states, const int64_t *__restrict__ slots,
-                           int64_t n, float alpha) {
-    __shared__ int64_t s_slot[kU];
-    __shared__ int64_t s_off[kU];   // slot * elems
-    __shared__ int s_prev[kU];      // latest earlier position of the same slot in the batch, or -1
-    __shared__ int s_last[kU];      // no later position of the batch has the same slot
-    __shared__ int s_dups;
-    __shared__ float s_val[kU][kConsThreads];
-    const float keep = 1.f - alpha;
-    const int tid = threadIdx.x;
-    const int64_t e = static_cast<int64_t>(blockIdx.x) * kConsThreads + tid;
-    for (int64_t c0 = 0; c0 < n; c0 += kU) {
-        __syncthreads();                       // the previous batch is done with s_*
-        if (tid < kU) {
-            const int64_t c = c0 + tid;
-            int64_t sl = c < n ? slots[c] : -1;
-            if (sl >= n_slots) {
-                if (blockIdx.x == 0) atomicOr(&g_smc_status, PRECOG_DEV_BAD_INDEX);
-                sl = -1;
-            }
-            if (sl < -1) sl = -1;
-            s_slot[tid] = sl;
-            s_off[tid] = sl >= 0 ? sl * elems : 0;
+struct BatchMeta {
+    int64_t off[kU];      // slot * elems (valid deposits)
+    int prev[kU];         // latest earlier position of the same slot, or -1
+    uint32_t valid;       // bit j: deposit j has a slot
+    uint32_t last;        // bit j: no later deposit of the batch has the same slot
+    uint32_t dups;        // some deposit repeats an earlier slot of the batch
+};
+
+__device__ __forceinline__ void describe_batch(BatchMeta &m, const int64_t *__restrict__ slots, int64_t c0,
+                                               int64_t n, int64_t n_slots, int64_t elems, int lane) {
+    int64_t sl = INT64_MIN;                       // lanes beyond the batch never match
+    if (lane < kU) {
+        const int64_t c = c0 + lane;
+        sl = c < n ? slots[c] : -1;
+        if (sl >= n_slots) {
+            atomicOr(&g_smc_status, PRECOG_DEV_BAD_INDEX);
+            sl = -1;
         }
-        if (tid == 0) s_dups = 0;
-        __syncthreads();
-        if (tid < kU) {
-            const int64_t sl = s_slot[tid];
-            int prev = -1, last = 1;
-            if (sl >= 0) {
-                for (int i = 0; i < tid; ++i)
-                    if (s_slot[i] == sl) prev = i;
-                for (int i = tid + 1; i < kU; ++i)
-                    if (s_slot[i] == sl) last = 0;
-            }
-            s_prev[tid] = prev;
-            s_last[tid] = last;
-            if (prev >= 0) atomicOr(&s_dups, 1);
-        }
-        __syncthreads();
-        if (e >= elems) continue;
-        float h[kU], v[kU];
-#pragma unroll
-        for (int j = 0; j < kU; ++j) {
-            h[j] = 0.f;
-            v[j] = 0.f;
-            if (s_slot[j] >= 0) h[j] = to_f32(states[(c0 + j) * elems + e]);
-        }
-#pragma unroll
-        for (int j = 0; j < kU; ++j)
-            if (s_slot[j] >= 0 && s_prev[j] < 0) v[j] = sem[s_off[j] + e];
-        if (!s_dups) {
-#pragma unroll
-            for (int j = 0; j < kU; ++j) v[j] = fmaf(keep, v[j], alpha * h[j]);
-        } else {
-#pragma unroll
-            for (int j = 0; j < kU; ++j) {
-                if (s_slot[j] < 0) continue;
-                const int pj = s_prev[j];
-                const float base = pj >= 0 ? s_val[pj][tid] : v[j];
-                v[j] = fmaf(keep, base, alpha * h[j]);
-                s_val[j][tid] = v[j];
-            }
-        }
-#pragma unroll
-        for (int j = 0; j < kU; ++j)
-            if (s_slot[j] >= 0 && s_last[j]) sem[s_off[j] + e] = v[j];
+        if (sl < -1) sl = -1;
+    }
+    const bool valid = lane < kU && sl >= 0;
+    const uint32_t same = __match_any_sync(0xffffffffu, sl);
+    const uint32_t below = same & ((1u << lane) - 1u);
+    const uint32_t above = lane == 31 ? 0u : (same & ~((2u << lane) - 1u));
+    const int prev = valid && below ? 31 - __clz(below) : -1;
+    const uint32_t vmask = __ballot_sync(0xffffffffu, valid);
+    const uint32_t lmask = __ballot_sync(0xffffffffu, valid && above == 0u);
+    const uint32_t dmask = __ballot_sync(0xffffffffu, prev >= 0);
+    if (lane < kU) {
+        m.off[lane] = valid ? sl * elems : 0;
+        m.prev[lane] = prev;
+    }
+    if (lane == 0) {
+        m.valid = vmask;
+        m.last = lmask;
+        m.dups = dmask != 0u;
     }
 }
 
-int sm_count() {
-    static int sms = 0;
-    if (sms == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        if (sms <= 0) sms = 1;
+template <typename TS, int VEC>
+__device__ __forceinline__ void load_state_vec(const TS *p, float (&h)[VEC]) {
+    if constexpr (VEC == 1) {
+        h[0] = to_f32(p[0]);
+    } else if constexpr (std::is_same<TS, float>::value) {
+        const float2 v = *reinterpret_cast<const float2 *>(p);
+        h[0] = v.x;
+        h[1] = v.y;
+    } else {
+        const uint32_t w = *reinterpret_cast<const uint32_t *>(p);
+        h[0] = __uint_as_float(w << 16);
+        h[1] = __uint_as_float(w & 0xffff0000u);
     }
-    return sms;
+}
+
+template <int VEC>
+__device__ __forceinline__ void load_sem(const float *p, float (&v)[VEC]) {
+    if constexpr (VEC == 1) {
+        v[0] = p[0];
+    } else {
+        const float2 q = *reinterpret_cast<const float2 *>(p);
+        v[0] = q.x;
+        v[1] = q.y;
+    }
+}
+
+template <int VEC>
+__device__ __forceinline__ void store_sem(float *p, const float (&v)[VEC]) {
+    if constexpr (VEC == 1) p[0] = v[0];
+    else *reinterpret_cast<float2 *>(p) = make_float2(v[0], v[1]);
+}
+
+template <typename TS, int VEC>
+__global__ void __launch_bounds__(kConsThreads)
+    smc_consolidate_kernel(float *__restrict__ sem, int64_t n_slots, int64_t elems,
+                           const TS *__restrict__ states, const int64_t *__restrict__ slots,
+                           int64_t n, float alpha) {
+    __shared__ BatchMeta s_meta[2];
+    __shared__ float s_val[kU][VEC][kConsThreads];
+    const float keep = 1.f - alpha;
+    const int tid = threadIdx.x, lane = tid & 31;
+    const int64_t e = (static_cast<int64_t>(blockIdx.x) * kConsThreads + tid) * VEC;
+    const bool mine = e < elems;
+    const int64_t nbatch = (n + kU - 1) / kU;
+    if (tid < 32) describe_batch(s_meta[0], slots, 0, n, n_slots, elems, lane);
+    __syncthreads();
+    for (int64_t b = 0; b < nbatch; ++b) {
+        const BatchMeta &m = s_meta[b & 1];
+        const int64_t c0 = b * kU;
+        float h[kU][VEC], v[kU][VEC];
+        if (mine) {
+#pragma unroll
+            for (int j = 0; j < kU; ++j) {
+#pragma unroll
+                for (int i = 0; i < VEC; ++i) h[j][i] = v[j][i] = 0.f;
+                if (m.valid >> j & 1u) load_state_vec<TS, VEC>(states + (c0 + j) * elems + e, h[j]);
+            }
+#pragma unroll
+            for (int j = 0; j < kU; ++j)
+                if ((m.valid >> j & 1u) && m.prev[j] < 0) load_sem<VEC>(sem + m.off[j] + e, v[j]);
+        }
+        // the next batch's description overlaps this batch's loads
+        if (tid < 32 && b + 1 < nbatch)
+            describe_batch(s_meta[(b + 1) & 1], slots, c0 + kU, n, n_slots, elems, lane);
+        if (mine) {
+            if (!m.dups) {
+#pragma unroll
+                for (int j = 0; j < kU; ++j)
+#pragma unroll
+                    for (int i = 0; i < VEC; ++i) v[j][i] = fmaf(keep, v[j][i], alpha * h[j][i]);
+            } else {
+#pragma unroll
+                for (int j = 0; j < kU; ++j) {
+                    if (!(m.valid >> j & 1u)) continue;
+                    const int pj = m.prev[j];
+#pragma unroll
+                    for (int i = 0; i < VEC; ++i) {
+                        const float base = pj >= 0 ? s_val[pj][i][tid] : v[j][i];
+                        v[j][i] = fmaf(keep, base, alpha * h[j][i]);
+                        s_val[j][i][tid] = v[j][i];
+                    }
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < kU; ++j)
+                if (m.last >> j & 1u) store_sem<VEC>(sem + m.off[j] + e, v[j]);
+        }
+        __syncthreads();   // the next batch's description is complete; this one may be rewritten
+    }
 }
 
 }  // namespace
@@ -198,15 +248,21 @@ cudaError_t launch_smc_consolidate(float *sem, int64_t n_slots, int64_t elems, c
                                    int states_dtype, const int64_t *slots, int64_t n, float alpha,
                                    cudaStream_t stream) {
     if (n == 0 || elems == 0) return cudaSuccess;
-    const int64_t blocks = (elems + kConsThreads - 1) / kConsThreads;
+    // pairs of elements when every row start stays 8-byte (fp32) / 4-byte (bf16) aligned
+    const bool pairs = elems % 2 == 0;
+    const int vec = pairs ? 2 : 1;
+    const int64_t blocks = (elems / vec + kConsThreads - 1) / kConsThreads;
     if (blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
     const unsigned grid = static_cast<unsigned>(blocks);
-    if (states_dtype == PRECOG_BF16)
-        smc_consolidate_kernel<__nv_bfloat16><<<grid, kConsThreads, 0, stream>>>(
-            sem, n_slots, elems, static_cast<const __nv_bfloat16 *>(states), slots, n, alpha);
-    else
-        smc_consolidate_kernel<float><<<grid, kConsThreads, 0, stream>>>(
-            sem, n_slots, elems, static_cast<const float *>(states), slots, n, alpha);
+    if (states_dtype == PRECOG_BF16) {
+        const auto *st = static_cast<const __nv_bfloat16 *>(states);
+        if (pairs) smc_consolidate_kernel<__nv_bfloat16, 2><<<grid, kConsThreads, 0, stream>>>(sem, n_slots, elems, st, slots, n, alpha);
+        else smc_consolidate_kernel<__nv_bfloat16, 1><<<grid, kConsThreads, 0, stream>>>(sem, n_slots, elems, st, slots, n, alpha);
+    } else {
+        const auto *st = static_cast<const float *>(states);
+        if (pairs) smc_consolidate_kernel<float, 2><<<grid, kConsThreads, 0, stream>>>(sem, n_slots, elems, st, slots, n, alpha);
+        else smc_consolidate_kernel<float, 1><<<grid, kConsThreads, 0, stream>>>(sem, n_slots, elems, st, slots, n, alpha);
+    }
     cudaError_t e = cudaGetLastError();
     if (e == cudaSuccess) count_launches(1);
     return e;
