@@ -150,6 +150,33 @@ class Clocks:
                 "power_w_max": max(power) if power else None, "samples": len(rows)}
 
 
+# ------------------------------------------------------------------------------ ranks
+
+
+def shard_seed(rank: int) -> int:
+    """Seed of a rank's corpus shard. Chunks are encoded independently (Sec. 4.2), so every
+    rank encodes its own chunks of the same shape: weak scaling, no exchange on the data
+    path."""
+    return 1000 * rank
+
+
+def reduce_max(v: float, world: int, device) -> float:
+    """The slowest rank's time (max over ranks); ``device`` is where the process group
+    reduces (a CUDA device under NCCL, the CPU under gloo)."""
+    if world == 1:
+        return v
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([v], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank_step: float, world: int, steps: int, seconds: float) -> float:
+    """Units processed by all ranks per second of the slowest rank."""
+    return world * units_per_rank_step * steps / seconds
+
+
 # ------------------------------------------------------------------------------ reference arm
 
 
@@ -384,15 +411,11 @@ def main():
             torch.distributed.barrier()
 
     def max_over_ranks(v):
-        if world == 1:
-            return v
-        t = torch.tensor([v], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        return float(t.item())
+        return reduce_max(v, world, dev)
 
     shape = synth.PAPER
     L, D, N = shape.n_layers, shape.D, shape.N
-    seed = 1000 * rank
+    seed = shard_seed(rank)
     off_np = synth.shape_offsets(shape, seed)
     T = int(off_np[-1])
     off = torch.from_numpy(off_np).to(dev)
@@ -470,7 +493,7 @@ def main():
     elapsed_ms = max_over_ranks(t0.elapsed_time(t1))
     scan_ms = [a.elapsed_time(b) for a, b in ev]
     tokens_per_step = T
-    value = world * tokens_per_step * args.steps / (elapsed_ms * 1e-3)
+    value = whole_job_rate(tokens_per_step, world, args.steps, elapsed_ms * 1e-3)
     ms_per_step = elapsed_ms / args.steps
 
     hbm, peak_src = peaks()
@@ -567,7 +590,7 @@ def main():
         torch.cuda.synchronize()
         e2e_s = max_over_ranks(time.perf_counter() - w0)
         barrier()
-        e2e = {"value": world * tokens_per_step * args.e2e_steps / e2e_s, "unit": UNIT,
+        e2e = {"value": whole_job_rate(tokens_per_step, world, args.e2e_steps, e2e_s), "unit": UNIT,
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                "ms_per_step": 1e3 * e2e_s / args.e2e_steps, "steps": args.e2e_steps}
         del host, hq, bank_host, out_host

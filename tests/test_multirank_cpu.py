@@ -1,0 +1,62 @@
+"""The multi-rank host logic of bench.py on CPU: two gloo ranks on 127.0.0.1. Each rank
+encodes its own corpus shard (different chunks, same shape; no exchange on the data path),
+the timed region is the slowest rank's time, and the reported rate counts the units of all
+ranks. No GPU is touched."""
+import os
+import socket
+
+import pytest
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, queue):
+    import torch
+    import torch.distributed as dist
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        import bench
+        import synth
+        seed = bench.shard_seed(rank)
+        inp = synth.device_scan_inputs(64, 16, 16, seed, 0, torch.device("cpu"), with_C=False)
+        x = inp["x"].float()
+        gathered = [torch.empty_like(x) for _ in range(world)]
+        dist.all_gather(gathered, x)
+        distinct = not torch.equal(gathered[0], gathered[1])
+        slowest = bench.reduce_max(1.0 + rank, world, torch.device("cpu"))
+        rate = bench.whole_job_rate(1000, world, 5, slowest)
+        queue.put((rank, seed, distinct, slowest, rate, tuple(x.shape)))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_gloo_ranks_shard_and_reduce():
+    mp = pytest.importorskip("torch.multiprocessing")
+    ctx = mp.get_context("spawn")
+    queue = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_rank_main, args=(r, 2, port, queue)) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(timeout=180)
+    assert all(p.exitcode == 0 for p in procs), [p.exitcode for p in procs]
+    res = sorted(queue.get(timeout=10) for _ in range(2))
+    (r0, s0, d0, t0, v0, sh0), (r1, s1, d1, t1, v1, sh1) = res
+    assert (r0, r1) == (0, 1) and s0 != s1            # each rank its own shard
+    assert sh0 == sh1 and d0 and d1                   # same shape, different chunks
+    assert t0 == t1 == 2.0                            # both ranks report the slowest time
+    assert v0 == v1 == 2 * 1000 * 5 / 2.0             # units of all ranks / slowest time
+
+
+def test_single_rank_helpers():
+    import bench
+    assert bench.shard_seed(0) == 0 and bench.shard_seed(3) == 3000
+    assert bench.reduce_max(4.5, 1, None) == 4.5
+    assert bench.whole_job_rate(10, 1, 3, 2.0) == 15.0
