@@ -740,6 +740,21 @@ int pick_slice(int D, int sz, int cpt) {
     return 0;
 }
 
+// True when a full-width launch would have fewer CTAs than the device has SMs.
+bool few_items(const ScanParams &p) {
+    static int sms = 0;
+    if (sms == 0) {
+        int dev = 0, n = 0;
+        if (cudaGetDevice(&dev) == cudaSuccess &&
+            cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && n > 0)
+            sms = n;
+        else
+            return false;
+    }
+    const int64_t slices = (p.D + kMaxSlice - 1) / kMaxSlice;
+    return static_cast<int64_t>(p.n_layers) * p.n_chunks * slices < sms;
+}
+
 template <class C>
 cudaError_t launch_cfg(const ScanParams &p, cudaStream_t stream) {
     const int DS = pick_slice(p.D, C::SZ, C::CPT);
@@ -779,6 +794,11 @@ cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
                               PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB>>(p, stream);
     } else {
         if constexpr (MODE == kPower) {
+            // Fewer work items than SMs (a single query's prefill: one CTA per layer) is a
+            // latency-bound launch: two channels per thread halve each thread's serial work
+            // per token (measured 27 -> 21 us for 24 layers x 64 tokens).
+            if (few_items(p))
+                return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, 2, 16, 2, 3>>(p, stream);
             return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, PRECOG_DIRECT_CPT, PRECOG_DIRECT_TILE,
                                   PRECOG_DIRECT_STAGES, PRECOG_DIRECT_MINB>>(p, stream);
         } else {
