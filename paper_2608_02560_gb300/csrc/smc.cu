@@ -94,12 +94,18 @@ struct BatchMeta {
     uint32_t dups;        // some deposit repeats an earlier slot of the batch
 };
 
-__device__ __forceinline__ void describe_batch(BatchMeta &m, const int64_t *__restrict__ slots, int64_t c0,
-                                               int64_t n, int64_t n_slots, int64_t elems, int lane) {
+// Lane j < kU of warp 0 reads deposit c0 + j's slot (-1 past the end); the reads
+// run two batches ahead of their use so that their latency is hidden.
+__device__ __forceinline__ int64_t read_slot(const int64_t *__restrict__ slots, int64_t c0, int64_t n, int lane) {
+    const int64_t c = c0 + lane;
+    return lane < kU && c < n ? slots[c] : -1;
+}
+
+__device__ __forceinline__ void describe_batch(BatchMeta &m, int64_t raw, int64_t n_slots, int64_t elems,
+                                               int lane) {
     int64_t sl = INT64_MIN;                       // lanes beyond the batch never match
     if (lane < kU) {
-        const int64_t c = c0 + lane;
-        sl = c < n ? slots[c] : -1;
+        sl = raw;
         if (sl >= n_slots) {
             atomicOr(&g_smc_status, PRECOG_DEV_BAD_INDEX);
             sl = -1;
@@ -169,26 +175,47 @@ __global__ void __launch_bounds__(kConsThreads)
     const int64_t e = (static_cast<int64_t>(blockIdx.x) * kConsThreads + tid) * VEC;
     const bool mine = e < elems;
     const int64_t nbatch = (n + kU - 1) / kU;
-    if (tid < 32) describe_batch(s_meta[0], slots, 0, n, n_slots, elems, lane);
+    // The deposits' states do not depend on the semantic table, so each batch's state
+    // loads are issued one batch ahead (every deposit that exists, slot or not).
+    auto load_states = [&](int64_t c0, float (&h)[kU][VEC]) {
+#pragma unroll
+        for (int j = 0; j < kU; ++j) {
+#pragma unroll
+            for (int i = 0; i < VEC; ++i) h[j][i] = 0.f;
+            if (mine && c0 + j < n) load_state_vec<TS, VEC>(states + (c0 + j) * elems + e, h[j]);
+        }
+    };
+    float h[kU][VEC];
+    load_states(0, h);
+    int64_t raw_next = 0;
+    if (tid < 32) {
+        const int64_t raw0 = read_slot(slots, 0, n, lane);
+        raw_next = read_slot(slots, kU, n, lane);
+        describe_batch(s_meta[0], raw0, n_slots, elems, lane);
+    }
     __syncthreads();
     for (int64_t b = 0; b < nbatch; ++b) {
         const BatchMeta &m = s_meta[b & 1];
         const int64_t c0 = b * kU;
-        float h[kU][VEC], v[kU][VEC];
+        float v[kU][VEC];
         if (mine) {
+            // first touch of each slot in this batch: after the previous batch's stores
+            // (same thread, program order)
 #pragma unroll
             for (int j = 0; j < kU; ++j) {
 #pragma unroll
-                for (int i = 0; i < VEC; ++i) h[j][i] = v[j][i] = 0.f;
-                if (m.valid >> j & 1u) load_state_vec<TS, VEC>(states + (c0 + j) * elems + e, h[j]);
-            }
-#pragma unroll
-            for (int j = 0; j < kU; ++j)
+                for (int i = 0; i < VEC; ++i) v[j][i] = 0.f;
                 if ((m.valid >> j & 1u) && m.prev[j] < 0) load_sem<VEC>(sem + m.off[j] + e, v[j]);
+            }
         }
+        float hn[kU][VEC];
+        load_states(c0 + kU, hn);
         // the next batch's description overlaps this batch's loads
-        if (tid < 32 && b + 1 < nbatch)
-            describe_batch(s_meta[(b + 1) & 1], slots, c0 + kU, n, n_slots, elems, lane);
+        if (tid < 32 && b + 1 < nbatch) {
+            const int64_t raw = raw_next;
+            raw_next = read_slot(slots, c0 + 2 * kU, n, lane);
+            describe_batch(s_meta[(b + 1) & 1], raw, n_slots, elems, lane);
+        }
         if (mine) {
             if (!m.dups) {
 #pragma unroll
@@ -212,6 +239,10 @@ __global__ void __launch_bounds__(kConsThreads)
             for (int j = 0; j < kU; ++j)
                 if (m.last >> j & 1u) store_sem<VEC>(sem + m.off[j] + e, v[j]);
         }
+#pragma unroll
+        for (int j = 0; j < kU; ++j)
+#pragma unroll
+            for (int i = 0; i < VEC; ++i) h[j][i] = hn[j][i];
         __syncthreads();   // the next batch's description is complete; this one may be rewritten
     }
 }

@@ -179,3 +179,31 @@ def test_complex_unsupported_forms_are_rejected(cuda_device):
     with pytest.raises(pg.PrecogError):
         pg.precog_prefill_composed(ins, 1, T, bank, rows, sc, 2,
                                    state_out=torch.empty((1, 1, D, 16), dtype=torch.complex64, device=d))
+
+
+def test_complex_paper_shaped_launch_sampled(cuda_device):
+    """The launch the benchmark times: one paper-shaped layer (4096 chunks x 3000 tokens,
+    D=256, N=16, bf16 inputs and bf16 complex states, A = -(n+1) + i*pi*n); sampled chunks
+    against the oracle."""
+    import torch
+    pg = _pg()
+    d = cuda_device
+    shape = synth.PAPER
+    off_np = synth.fixed_offsets(shape.n_chunks, shape.chunk_len)
+    T = int(off_np[-1])
+    inp = synth.device_scan_inputs(T, shape.D, shape.N, 0, 0, d, with_C=False)
+    im = (np.pi * torch.arange(shape.N, device=d, dtype=torch.float32)).expand(shape.D, shape.N)
+    A = torch.complex(inp["A"], im).contiguous()
+    st = torch.empty((shape.n_chunks, 1, shape.D, shape.N, 2), dtype=torch.bfloat16, device=d)
+    ins = pg.scan_inputs(inp["x"], inp["dt"], inp["B"], A, a_kind=pg.PRECOG_A_COMPLEX)
+    pg.precog_encode_chunks(ins, torch.from_numpy(off_np).to(d), T, states_out=st)
+    assert pg.precog_device_status()[0] == 0
+    An = A.cpu().numpy()
+    for c in (0, 1777, shape.n_chunks - 1):
+        s = int(off_np[c])
+        sl = slice(s, s + shape.chunk_len)
+        ref, _ = oracle.scan_complex(to_np(inp["x"][sl]), to_np(inp["dt"][sl]), An.real, An.imag,
+                                     to_np(inp["B"][sl]), [0, shape.chunk_len])
+        f = st[c, 0].float().cpu().numpy().astype(np.float64)
+        assert rel_err_stored(f[..., 0], ref[0].real) < TOL_BF16, c
+        assert rel_err_stored(f[..., 1], ref[0].imag) < TOL_BF16, c

@@ -120,3 +120,47 @@ def test_consolidate_flags_slot_outside_table(cuda_device):
     keep[2] = -1
     ref = oracle.smc_consolidate(sem0, states, keep, 0.5)
     assert rel_err(to_np(sem), ref) < TOL_F32
+
+
+def test_smc_benchmark_sizes_sampled(cuda_device):
+    """The launches the benchmark times: 4096 chunk embeddings (fp16, dim 768) routed over
+    16 domains x 64 sub-clusters, and 4096 bf16 24-layer states folded into 64 slots.
+    Routing is compared where the oracle's best score leads the runner-up by more than
+    fp32 error can move (both levels); consolidation on sampled state elements."""
+    import torch
+    import paper_2608_02560_gb300 as pg
+    d = cuda_device
+    n, Md, J, dim = 4096, 16, 64, synth.QUERY_DIM
+    index = synth.device_unit_index(n + Md + Md * J, dim, 21, d)
+    emb, dom = index[:n], index[n:n + Md].contiguous()
+    sub = index[n + Md:].contiguous().view(Md, J, dim)
+    Jt = torch.full((Md,), J, dtype=torch.int32, device=d)
+    om = torch.empty(n, dtype=torch.int32, device=d)
+    oj = torch.empty(n, dtype=torch.int32, device=d)
+    osl = torch.empty(n, dtype=torch.int64, device=d)
+    pg.precog_smc_route(emb, dom, sub, Jt, om, oj, osl)
+    assert pg.precog_device_status()[0] == 0
+    E, P, S = (to_np(t) for t in (emb, dom, sub))
+    rm, rj = oracle.smc_route(E, P, S, Jt.cpu().numpy())
+    sd = E @ P.T
+    top2 = np.sort(sd, axis=1)[:, -2:]
+    ok_m = (top2[:, 1] - top2[:, 0]) > 1e-4
+    ss = np.einsum("nd,njd->nj", E, S[rm])
+    top2j = np.sort(ss, axis=1)[:, -2:]
+    ok_j = ok_m & ((top2j[:, 1] - top2j[:, 0]) > 1e-4)
+    assert ok_j.sum() > n // 2
+    np.testing.assert_array_equal(om.cpu().numpy()[ok_m], rm[ok_m])
+    np.testing.assert_array_equal(oj.cpu().numpy()[ok_j], rj[ok_j])
+    # consolidation of 4096 24-layer states into 64 slots, in deposit order
+    L, D, N = 24, 256, 16
+    states = synth.device_normal_bank(n, L * D * N, 22, d)
+    slots = torch.arange(n, dtype=torch.int64, device=d) * 7 % 64
+    sem0 = torch.zeros((64, L * D * N), dtype=torch.float32, device=d)
+    sem = sem0.clone()
+    pg.precog_smc_consolidate(sem, states, slots, 0.1)
+    assert pg.precog_device_status()[0] == 0
+    cols = torch.from_numpy(np.random.default_rng(3).choice(L * D * N, size=257, replace=False)).to(d)
+    ref = oracle.smc_consolidate(to_np(sem0[:, cols]), to_np(states[:, cols]), slots.cpu().numpy(), 0.1)
+    got = to_np(sem[:, cols])
+    for s in range(64):
+        assert rel_err(got[s], ref[s]) < TOL_F32, s
