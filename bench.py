@@ -61,7 +61,8 @@ def parse_args():
     ap.add_argument("--no-latency", action="store_true")
     ap.add_argument("--no-extras", action="store_true",
                     help="skip the measurements of the extension rows (top-k, trajectory, complex A, SMC)")
-    ap.add_argument("--case", choices=["full", "scan-small", "retrieve-small", "topk-small", "prefill-small"],
+    ap.add_argument("--case", choices=["full", "scan-small", "retrieve-small", "topk-small", "prefill-small",
+                                       "wide-encode", "wide-encode-y", "ragged-encode"],
                     default="full",
                     help="small single-kernel cases (a few GB) used for profiler captures")
     return ap.parse_args()
@@ -247,6 +248,26 @@ def run_case(args):
         fn = lambda: pg.precog_encode_chunks(si, off, T, states_out=bank, layer0=0, L_total=shape.n_layers)
         res["algorithmic_bytes_per_launch"] = scan_bytes_per_launch(T, chunks, shape.D, shape.N)
         res["scale_to_full_launch"] = shape.n_chunks * shape.chunk_len / T
+    elif args.case in ("wide-encode", "wide-encode-y", "ragged-encode"):
+        # one layer of the single-layer wide encode (D=2048, 1024 x 512 tokens; capture or
+        # readout) or of the ragged encode (D=512, 8192 chunks of 256..4096 tokens)
+        shape = synth.RAGGED if args.case == "ragged-encode" else synth.WIDE
+        y_mode = args.case == "wide-encode-y"
+        off_np = synth.shape_offsets(shape, 0)
+        T = int(off_np[-1])
+        inp = synth.device_scan_inputs(T, shape.D, shape.N, 0, 0, dev, with_C=y_mode)
+        off = torch.from_numpy(off_np).to(dev)
+        sdt = torch.float32 if shape is synth.WIDE else torch.bfloat16
+        bank = torch.empty((shape.n_chunks, 1, shape.D, shape.N), dtype=sdt, device=dev)
+        y = torch.empty((1, T, shape.D), dtype=torch.bfloat16, device=dev) if y_mode else None
+        si = pg.scan_inputs(inp["x"], inp["dt"], inp["B"], inp["A"], inp["C"] if y_mode else None,
+                            a_kind=pg.PRECOG_A_POWER)
+        fn = lambda: pg.precog_encode_chunks(si, off, T, states_out=bank, y_out=y)
+        nb = scan_bytes_per_launch(T, shape.n_chunks, shape.D, shape.N, state_bytes=bank.element_size())
+        if y_mode:
+            nb += T * shape.N * 2 + T * shape.D * 2
+        res["algorithmic_bytes_per_launch"] = nb
+        res["tokens"] = T
     elif args.case in ("retrieve-small", "topk-small"):
         M = 1 << 18
         index = synth.device_unit_index(M, synth.QUERY_DIM, 0, dev)
@@ -277,6 +298,10 @@ def run_case(args):
         ev[2 * i + 1].record()
     torch.cuda.synchronize()
     res["ms"] = [ev[2 * i].elapsed_time(ev[2 * i + 1]) for i in range(3)]
+    if args.case in ("wide-encode", "wide-encode-y", "ragged-encode"):
+        best = min(res["ms"][1:])
+        res["achieved_gbs"] = res["algorithmic_bytes_per_launch"] / (best * 1e-3) / 1e9
+        res["frac_hbm"] = res["achieved_gbs"] / peaks()[0]
     st, bits = pg.precog_device_status()
     res["device_status"] = [st, bits]
     print(json.dumps(res), flush=True)

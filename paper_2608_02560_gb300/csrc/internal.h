@@ -3,6 +3,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 namespace precog {
@@ -46,6 +47,12 @@ struct ScanParams {
     int64_t traj_stride;
     const int64_t *traj_offsets;  // [n_chunks+1] first entry of each chunk
 };
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point (no link against
+// libcuda); false if the entry point is missing or the driver rejects the map.
+bool encode_tiled_map(CUtensorMap *map, CUtensorMapDataType dtype, cuuint32_t rank, const void *base,
+                      const cuuint64_t *dims, const cuuint64_t *strides_bytes, const cuuint32_t *box,
+                      CUtensorMapSwizzle swizzle);
 
 // Kernel launches made by this library since the process started.
 void count_launches(uint64_t n);

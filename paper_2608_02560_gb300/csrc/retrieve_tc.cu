@@ -311,36 +311,37 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-using EncodeTiled = PFN_cuTensorMapEncodeTiled_v12000;
-
-EncodeTiled encode_fn() {
-    static EncodeTiled fn = nullptr;
-    if (fn == nullptr) {
-        void *p = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                             &q) == cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiled>(p);
-    }
-    return fn;
-}
-
 bool make_map(CUtensorMap *map, const void *base, int64_t rows, int dim, bool bf16, int box_rows) {
-    EncodeTiled fn = encode_fn();
-    if (fn == nullptr) return false;
     const cuuint64_t gdim[2] = {static_cast<cuuint64_t>(dim), static_cast<cuuint64_t>(rows)};
     const cuuint64_t gstride[1] = {static_cast<cuuint64_t>(dim) * 2};
     const cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), static_cast<cuuint32_t>(box_rows)};
-    const cuuint32_t estride[2] = {1, 1};
-    const CUresult r = fn(map, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16,
-                          2, const_cast<void *>(base), gdim, gstride, box, estride,
-                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS;
+    return encode_tiled_map(map, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2,
+                            base, gdim, gstride, box, CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
 }  // namespace
+
+using EncodeTiled = PFN_cuTensorMapEncodeTiled_v12000;
+
+bool encode_tiled_map(CUtensorMap *map, CUtensorMapDataType dtype, cuuint32_t rank, const void *base,
+                      const cuuint64_t *dims, const cuuint64_t *strides_bytes, const cuuint32_t *box,
+                      CUtensorMapSwizzle swizzle) {
+    static EncodeTiled fn = [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            return reinterpret_cast<EncodeTiled>(p);
+        return static_cast<EncodeTiled>(nullptr);
+    }();
+    if (fn == nullptr) return false;
+    const cuuint32_t estride[5] = {1, 1, 1, 1, 1};
+    const CUresult r = fn(map, dtype, rank, const_cast<void *>(base), dims, strides_bytes, box, estride,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
 
 size_t retrieve_tc_smem_bytes() { return sizeof(Smem) + 1024; }
 

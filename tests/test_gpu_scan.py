@@ -139,6 +139,40 @@ def test_multi_layer_call_and_layer_offset(cuda_device):
             assert rel_err(got[c, 2 + l], ref[c]) < TOL_F32
 
 
+@pytest.mark.parametrize("D,y_mode", [(512, False), (512, True), (768, True)])
+def test_multi_layer_sliced_channels(cuda_device, D, y_mode):
+    """Channels wider than one CTA's 256-channel slice, three layers in one call: each CTA
+    stages its slice of x and dt through a 3-D tensor map (channel, row, layer); chunks
+    end inside and at the end of 16-row tiles. Every layer's states (and y) vs the oracle."""
+    import torch
+    pg = _pg()
+    d = cuda_device
+    L, N = 3, 16
+    off = np.array([0, 1, 17, 17, 53, 200], dtype=np.int64)
+    T = int(off[-1])
+    ins = [synth.host_scan_inputs(T, D, N, seed=90 + l) for l in range(L)]
+    st = lambda k: _t(np.stack([i[k] for i in ins]), d)
+    x, dt, B, C = st(0), st(1), st(3), st(4)
+    A = _t(np.stack([synth.structured_A(D, N) * (1 + 0.25 * l) for l in range(L)]), d)
+    n = len(off) - 1
+    bank = torch.full((n, L, D, N), float("nan"), dtype=torch.float32, device=d)
+    y = torch.full((L, T, D), float("nan"), dtype=torch.float32, device=d) if y_mode else None
+    pg.precog_encode_chunks(pg.scan_inputs(x, dt, B, A, C if y_mode else None, a_kind=pg.PRECOG_A_POWER),
+                            _t(off, d, torch.int64), T, states_out=bank, y_out=y)
+    assert pg.precog_device_status()[0] == 0
+    got = to_np(bank)
+    for l in range(L):
+        ref, ref_y = oracle.scan(ins[l][0], ins[l][1], synth.structured_A(D, N) * (1 + 0.25 * l),
+                                 ins[l][3], off, C=ins[l][4] if y_mode else None, want_y=y_mode)
+        for c in range(n):
+            if off[c] == off[c + 1]:
+                assert np.all(got[c, l] == 0)
+            else:
+                assert rel_err(got[c, l], ref[c]) < TOL_F32
+        if y_mode:
+            assert rel_err(to_np(y[l]), ref_y) < TOL_F32
+
+
 def test_bf16_capture_and_readout(cuda_device):
     """bf16 inputs, fp32 accumulation: bf16 and fp32 state capture, bf16 readout."""
     import torch
