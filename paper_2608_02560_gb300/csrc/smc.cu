@@ -247,6 +247,90 @@ __global__ void __launch_bounds__(kConsThreads)
     }
 }
 
+// The same fold with one CTA per (slot, range of elements), for tables of few
+// slots: the CTA gathers its slot's deposits in deposit order (ballots over the
+// slot ids, kGather at a time), then streams their states with several deposits'
+// loads in flight, keeping its elements' semantic values in registers from the
+// first deposit to the last: each state element is read once and each semantic
+// element read and written once.
+constexpr int kSlotThreads = 256;
+constexpr int kSlotItems = 4;                    // element groups of VEC per thread
+constexpr int kGather = 4 * kSlotThreads;        // slot ids examined per gathering pass
+constexpr int kFoldAhead = 4;                    // deposits whose loads are in flight together
+
+template <typename TS, int VEC>
+__global__ void __launch_bounds__(kSlotThreads)
+    smc_consolidate_slot_kernel(float *__restrict__ sem, int64_t n_slots, int64_t elems,
+                                const TS *__restrict__ states, const int64_t *__restrict__ slots,
+                                int64_t n, float alpha) {
+    __shared__ int32_t s_list[kGather];
+    __shared__ int s_warp[kSlotThreads / 32];
+    __shared__ int s_total;
+    const int64_t slot = blockIdx.y;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const float keep = 1.f - alpha;
+    const bool flagger = blockIdx.x == 0 && blockIdx.y == 0;
+    int64_t e[kSlotItems];
+    float v[kSlotItems][VEC];
+#pragma unroll
+    for (int i = 0; i < kSlotItems; ++i) {
+        e[i] = ((static_cast<int64_t>(blockIdx.x) * kSlotItems + i) * kSlotThreads + tid) * VEC;
+        if (e[i] < elems) load_sem<VEC>(sem + slot * elems + e[i], v[i]);
+    }
+    for (int64_t c0 = 0; c0 < n; c0 += kGather) {
+        int64_t sl[4];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            const int64_t c = c0 + r * kSlotThreads + tid;
+            sl[r] = c < n ? slots[c] : -1;
+            if (flagger && sl[r] >= n_slots) atomicOr(&g_smc_status, PRECOG_DEV_BAD_INDEX);
+        }
+        if (tid == 0) s_total = 0;
+        __syncthreads();
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            const bool hit = sl[r] == slot;
+            const uint32_t ball = __ballot_sync(0xffffffffu, hit);
+            if (lane == 0) s_warp[warp] = __popc(ball);
+            __syncthreads();
+            int base = s_total;
+            for (int w = 0; w < warp; ++w) base += s_warp[w];
+            if (hit) s_list[base + __popc(ball & ((1u << lane) - 1u))] = static_cast<int32_t>(r * kSlotThreads + tid);
+            __syncthreads();
+            if (tid == 0)
+                for (int w = 0; w < kSlotThreads / 32; ++w) s_total += s_warp[w];
+            __syncthreads();
+        }
+        const int m = s_total;
+        for (int j0 = 0; j0 < m; j0 += kFoldAhead) {
+            float h[kFoldAhead][kSlotItems][VEC];
+#pragma unroll
+            for (int q = 0; q < kFoldAhead; ++q) {
+                const int j = j0 + q;
+                const int64_t c = j < m ? c0 + s_list[j] : 0;
+#pragma unroll
+                for (int i = 0; i < kSlotItems; ++i) {
+#pragma unroll
+                    for (int k = 0; k < VEC; ++k) h[q][i][k] = 0.f;
+                    if (j < m && e[i] < elems) load_state_vec<TS, VEC>(states + c * elems + e[i], h[q][i]);
+                }
+            }
+#pragma unroll
+            for (int q = 0; q < kFoldAhead; ++q) {
+                if (j0 + q >= m) break;
+#pragma unroll
+                for (int i = 0; i < kSlotItems; ++i)
+#pragma unroll
+                    for (int k = 0; k < VEC; ++k) v[i][k] = fmaf(keep, v[i][k], alpha * h[q][i][k]);
+            }
+        }
+        __syncthreads();   // s_list is rebuilt by the next pass
+    }
+#pragma unroll
+    for (int i = 0; i < kSlotItems; ++i)
+        if (e[i] < elems) store_sem<VEC>(sem + slot * elems + e[i], v[i]);
+}
+
 }  // namespace
 
 cudaError_t launch_smc_route(const void *emb, int dtype, int64_t n, int dim, const void *dom, int M,
@@ -285,6 +369,24 @@ cudaError_t launch_smc_consolidate(float *sem, int64_t n_slots, int64_t elems, c
     const int64_t blocks = (elems / vec + kConsThreads - 1) / kConsThreads;
     if (blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
     const unsigned grid = static_cast<unsigned>(blocks);
+    // Few slots: one CTA per (slot, element range). Each CTA reads all n slot ids (from
+    // L2), n_slots / 512 of the state bytes for bf16 states, so it pays up to 256 slots.
+    if (n_slots >= 1 && n_slots <= 256) {
+        const int64_t per_cta = static_cast<int64_t>(kSlotThreads) * kSlotItems * vec;
+        const dim3 g2(static_cast<unsigned>((elems + per_cta - 1) / per_cta), static_cast<unsigned>(n_slots));
+        if (states_dtype == PRECOG_BF16) {
+            const auto *st = static_cast<const __nv_bfloat16 *>(states);
+            if (pairs) smc_consolidate_slot_kernel<__nv_bfloat16, 2><<<g2, kSlotThreads, 0, stream>>>(sem, n_slots, elems, st, slots, n, alpha);
+            else smc_consolidate_slot_kernel<__nv_bfloat16, 1><<<g2, kSlotThreads, 0, stream>>>(sem, n_slots, elems, st, slots, n, alpha);
+        } else {
+            const auto *st = static_cast<const float *>(states);
+            if (pairs) smc_consolidate_slot_kernel<float, 2><<<g2, kSlotThreads, 0, stream>>>(sem, n_slots, elems, st, slots, n, alpha);
+            else smc_consolidate_slot_kernel<float, 1><<<g2, kSlotThreads, 0, stream>>>(sem, n_slots, elems, st, slots, n, alpha);
+        }
+        cudaError_t e = cudaGetLastError();
+        if (e == cudaSuccess) count_launches(1);
+        return e;
+    }
     if (states_dtype == PRECOG_BF16) {
         const auto *st = static_cast<const __nv_bfloat16 *>(states);
         if (pairs) smc_consolidate_kernel<__nv_bfloat16, 2><<<grid, kConsThreads, 0, stream>>>(sem, n_slots, elems, st, slots, n, alpha);

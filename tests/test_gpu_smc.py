@@ -75,11 +75,13 @@ def test_consolidate_then_session_init(cuda_device):
 
 
 @pytest.mark.parametrize("n,n_slots,pattern", [(200, 64, "cyclic"), (77, 3, "runs"), (1, 5, "cyclic"),
-                                               (96, 40, "random")])
+                                               (96, 40, "random"), (2500, 7, "random"),
+                                               (500, 300, "random"), (700, 1000, "runs")])
 def test_consolidate_deposit_patterns(cuda_device, n, n_slots, pattern):
-    """Deposit orders that exercise the batched fold: no slot repeated within a batch
-    (cyclic), long runs of one slot, a single deposit, random slots with -1 mixed in;
-    fp32 states of an odd element count."""
+    """Deposit orders that exercise both folds (per-slot CTAs for tables of at most 256
+    slots, deposit batches beyond): no slot repeated within a batch (cyclic), long runs of
+    one slot, a single deposit, random slots with -1 mixed in, more deposits than one
+    gathering pass; fp32 states of an odd element count."""
     import torch
     import paper_2608_02560_gb300 as pg
     rng = np.random.default_rng(n + n_slots)
