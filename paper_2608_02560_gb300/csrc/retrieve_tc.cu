@@ -1,18 +1,22 @@
-// Top-1 retrieval for a batch of queries on the 5th-generation tensor cores
-// (Sec. 4.2 query-time retrieval, exact dot product, lowest row on ties).
+// Top-1 (and top-k) retrieval for a batch of queries on the 5th-generation tensor
+// cores (Sec. 4.2 query-time retrieval, exact dot product, lowest row on ties).
 //
 // S = Q K^T is a dense contraction once several queries share a pass over the
 // index, so it runs on tcgen05: queries are the A operand (up to two 128-row
-// halves), key rows the B operand (tiles of 128 rows), dim the K dimension in
-// blocks of 64 (128 bytes, 128B-swizzled). fp32 accumulators live in tensor
-// memory, double-buffered (2 tiles x 2 halves x 128 columns = all 512
-// columns), so the argmax of one tile overlaps the MMAs of the next. The
+// halves), key rows the B operand (tiles of 256 rows), dim the K dimension in
+// blocks of 64 (128 bytes, 128B-swizzled). The kernel is bound by what shared
+// memory can be filled with from L2 (about 10 TB/s over the chip), and the
+// query operand is re-read for every key tile, so the key tile is as wide as
+// one MMA allows (N = 256): 64 KB staged per 64-wide k-block for 2 x 128 x 256
+// x 64 multiply-adds. fp32 accumulators live in tensor memory: one query half
+// uses 256 columns and is double-buffered, so the argmax of one tile overlaps
+// the MMAs of the next; two halves fill all 512 columns with one buffer. The
 // score matrix never leaves the SM: thread q of the epilogue owns TMEM lane q
 // (one query) and scans its columns (key rows) in increasing order with a
 // strict '>', which keeps the lowest row on ties; NaN never compares greater.
 //
 // Warp roles (one persistent CTA per SM, 192 threads):
-//   warp 0  TMA producer: A (queries) and B (key tile) k-blocks into a 4-stage ring
+//   warp 0  TMA producer: A (queries) and B (key tile) k-blocks into a 3-stage ring
 //   warp 1  TMEM owner and MMA issuer (one elected lane)
 //   warps 2-5 epilogue: TMEM -> registers -> running (score, row) per query
 // Every wait is bounded; on expiry the CTA flags PRECOG_DEV_TIMEOUT and leaves
@@ -30,9 +34,9 @@ namespace {
 __device__ uint32_t g_retrieve_status_tc;
 
 constexpr int kBM = 128;          // queries per MMA (one half)
-constexpr int kBN = 128;          // key rows per tile
+constexpr int kBN = 256;          // key rows per tile
 constexpr int kBK = 64;           // dim per k-block (128 bytes of fp16/bf16)
-constexpr int kStages = 4;
+constexpr int kStages = 3;
 constexpr int kThreads = 192;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kABytes = kBM * kBK * 2;   // one query half per stage
@@ -66,7 +70,7 @@ __device__ __forceinline__ uint64_t sw128_desc(const void *tile) {
 }
 
 // Instruction descriptor, kind::f16: fp32 accumulate, A and B of the same
-// 16-bit type, both K-major, M = 128, N = 128.
+// 16-bit type, both K-major, M = 128, N = 256.
 __host__ __device__ constexpr uint32_t idesc_f16(bool bf16) {
     return (1u << 4)                                    // D: f32
            | ((bf16 ? 1u : 0u) << 7)                    // A type
@@ -123,6 +127,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const int nhalf = nq > kBM ? 2 : 1;
+    // accumulator columns: one query half x 256 keys = 256 columns, so a single half is
+    // double-buffered (the argmax of a tile overlaps the next tile's MMAs) and two halves
+    // fill all 512 columns with one buffer
+    const int nbuf = nhalf == 1 ? 2 : 1;
     const int nkb = (dim + kBK - 1) / kBK;
     const int64_t ntiles = (M + kBN - 1) / kBN;
 
@@ -180,11 +188,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             int it = 0;
             bool alive = true;
             for (int64_t tile = blockIdx.x; tile < ntiles && alive; tile += gridDim.x, ++it) {
-                const int acc = it & 1;
-                const uint32_t ause = static_cast<uint32_t>(it >> 1);
+                const int acc = it % nbuf;
+                const uint32_t ause = static_cast<uint32_t>(it / nbuf);
                 if (!wait_or_abort(&sm.acc_empty[acc], (ause & 1u) ^ 1u, sm)) break;
                 tc_fence_after();
-                const uint32_t d0 = tmem + static_cast<uint32_t>(acc * 2 * kBN);
+                const uint32_t d0 = tmem + static_cast<uint32_t>(acc * kBN);
                 for (int kb = 0; kb < nkb; ++kb, ++g) {
                     const int s = g % kStages;
                     if (!wait_or_abort(&sm.full[s], (g / kStages) & 1u, sm)) {
@@ -220,10 +228,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int j = 0; j < (LIST > 1 ? LIST : 1); ++j) lst[h][j] = 0ull;
         int it = 0;
         for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
-            const int acc = it & 1;
+            const int acc = it % nbuf;
             // one lane waits, the warp follows its verdict (tcgen05.ld needs the whole warp)
             bool ok = true;
-            if (lane == 0) ok = wait_or_abort(&sm.acc_full[acc], static_cast<uint32_t>(it >> 1) & 1u, sm);
+            if (lane == 0) ok = wait_or_abort(&sm.acc_full[acc], static_cast<uint32_t>(it / nbuf) & 1u, sm);
             ok = __shfl_sync(0xffffffffu, ok, 0);
             if (!ok) break;
             tc_fence_after();
@@ -233,7 +241,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int c0 = 0; c0 < kBN; c0 += 32) {
                     float v[32];
                     tmem_ld32(tmem + (static_cast<uint32_t>(quarter * 32) << 16) +
-                                  static_cast<uint32_t>(acc * 2 * kBN + h * kBN + c0),
+                                  static_cast<uint32_t>(acc * kBN + h * kBN + c0),
                               v);
                     const int64_t rbase = row0 + c0;
                     // Fast path: the column maximum of the 32 values (NaN ignored). Only
@@ -342,6 +350,8 @@ bool encode_tiled_map(CUtensorMap *map, CUtensorMapDataType dtype, cuuint32_t ra
                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
+
+static_assert(sizeof(Smem) + 1024 <= 227 * 1024, "the ring and scratch must fit one CTA's shared memory");
 
 size_t retrieve_tc_smem_bytes() { return sizeof(Smem) + 1024; }
 
