@@ -89,7 +89,7 @@ cudaError_t retrieve_tc_status_word_read_clear(uint32_t *bits);
 // Top-k retrieval (k <= 8): partial lists of 8 packed keys per (part, query).
 size_t retrieve_topk_workspace_size(int64_t M, int32_t dim, int32_t n_queries);
 cudaError_t launch_retrieve_topk(const RetrieveParams &p, int k, cudaStream_t stream);
-cudaError_t launch_retrieve_tc_topk(const RetrieveParams &p, int grid, cudaStream_t stream,
+cudaError_t launch_retrieve_tc_topk(const RetrieveParams &p, int k, int grid, cudaStream_t stream,
                                     uint64_t *launches);
 cudaError_t launch_retrieve(const RetrieveParams &p, cudaStream_t stream);
 cudaError_t retrieve_status_word_read_clear(uint32_t *bits);

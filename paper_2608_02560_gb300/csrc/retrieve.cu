@@ -462,7 +462,7 @@ cudaError_t launch_retrieve_topk(const RetrieveParams &p, int k, cudaStream_t st
     int parts;
     if (use_tc(p)) {
         parts = retrieve_tc_grid(p.M, num_sms());
-        e = launch_retrieve_tc_topk(p, parts, stream, &launches);
+        e = launch_retrieve_tc_topk(p, k, parts, stream, &launches);
     } else {
         parts = gemv_grid(p.M);
         switch (p.dtype) {

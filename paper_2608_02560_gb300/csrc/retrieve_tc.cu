@@ -37,6 +37,7 @@ constexpr int kBM = 128;          // queries per MMA (one half)
 constexpr int kBN = 256;          // key rows per tile
 constexpr int kBK = 64;           // dim per k-block (128 bytes of fp16/bf16)
 constexpr int kStages = 3;
+constexpr int kTopkStride = 8;    // keys per (CTA, query) in the top-k workspace
 constexpr int kThreads = 192;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kABytes = kBM * kBK * 2;   // one query half per stage
@@ -114,7 +115,9 @@ __device__ __forceinline__ unsigned long long tc_key(float s, int64_t row) {
 }
 
 // LIST = 1: partial[blockIdx.x * n_queries + q0 + q] = packed best key of this CTA.
-// LIST > 1: partial[(blockIdx.x * n_queries + q0 + q) * LIST + j] = its LIST best, sorted.
+// LIST > 1: partial[(blockIdx.x * n_queries + q0 + q) * kTopkStride + j] = its LIST best,
+// sorted, then zero keys ("no row") up to kTopkStride. A shorter list (the smallest of
+// 2, 4, 8 that holds k) raises the running threshold sooner and costs less per insertion.
 template <int LIST>
 __global__ void __launch_bounds__(kThreads, 1)
     retrieve_tc_kernel(const __grid_constant__ CUtensorMap tmap_q,
@@ -297,8 +300,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int q = h * kBM + qrow;
             if (LIST > 1 && q < nq) {
 #pragma unroll
-                for (int j = 0; j < (LIST > 1 ? LIST : 1); ++j)
-                    partial[(static_cast<int64_t>(blockIdx.x) * n_queries + q0 + q) * LIST + j] = lst[h][j];
+                for (int j = 0; j < kTopkStride; ++j)
+                    partial[(static_cast<int64_t>(blockIdx.x) * n_queries + q0 + q) * kTopkStride + j] =
+                        j < LIST ? lst[h][j < LIST ? j : 0] : 0ull;
             }
             if (LIST == 1 && q < nq) {
                 unsigned long long key = 0ull;
@@ -389,8 +393,10 @@ cudaError_t launch_retrieve_tc(const RetrieveParams &p, int grid, cudaStream_t s
     return launch_tc<1>(p, grid, stream, launches);
 }
 
-cudaError_t launch_retrieve_tc_topk(const RetrieveParams &p, int grid, cudaStream_t stream,
+cudaError_t launch_retrieve_tc_topk(const RetrieveParams &p, int k, int grid, cudaStream_t stream,
                                     uint64_t *launches) {
+    if (k <= 2) return launch_tc<2>(p, grid, stream, launches);
+    if (k <= 4) return launch_tc<4>(p, grid, stream, launches);
     return launch_tc<8>(p, grid, stream, launches);
 }
 
