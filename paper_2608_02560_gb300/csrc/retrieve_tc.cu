@@ -15,10 +15,12 @@
 // (one query) and scans its columns (key rows) in increasing order with a
 // strict '>', which keeps the lowest row on ties; NaN never compares greater.
 //
-// Warp roles (one persistent CTA per SM, 192 threads):
+// Warp roles (one persistent CTA per SM, 320 threads):
 //   warp 0  TMA producer: A (queries) and B (key tile) k-blocks into a 3-stage ring
 //   warp 1  TMEM owner and MMA issuer (one elected lane)
-//   warps 2-5 epilogue: TMEM -> registers -> running (score, row) per query
+//   warps 2-5 / 6-9 epilogue of query half 0 / 1: TMEM -> registers -> running
+//   (score, row) per query; with two halves the accumulators are single-buffered, so
+//   splitting the halves over two groups halves the time the MMAs wait for them
 // Every wait is bounded; on expiry the CTA flags PRECOG_DEV_TIMEOUT and leaves
 // through the same teardown (TMEM freed, issued copies drained).
 #include <cuda.h>
@@ -38,7 +40,7 @@ constexpr int kBN = 256;          // key rows per tile
 constexpr int kBK = 64;           // dim per k-block (128 bytes of fp16/bf16)
 constexpr int kStages = 3;
 constexpr int kTopkStride = 8;    // keys per (CTA, query) in the top-k workspace
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;     // 2 control warps + 8 epilogue warps
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kABytes = kBM * kBK * 2;   // one query half per stage
 constexpr uint32_t kBBytes = kBN * kBK * 2;
@@ -54,7 +56,7 @@ struct Smem {
     uint32_t tmem_base;
     uint32_t abort_flag;
     // epilogue scratch: one row of 32 scores per epilogue thread (padded: conflict-free)
-    float epi[4 * 32][33];
+    float epi[8 * 32][33];
 };
 
 // Shared-memory matrix descriptor: K-major operand, 128B swizzle, rows of 128
@@ -144,7 +146,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&sm.acc_full[a], 1);
-            mbar_init(&sm.acc_empty[a], 4 * 32);
+            mbar_init(&sm.acc_empty[a], nhalf * 4 * 32);   // the epilogue threads of the halves in use
         }
         sm.abort_flag = 0;
         fence_barrier_init();
@@ -219,27 +221,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
     } else {
         // ---------------- epilogue: argmax over key rows, per query ----------------
+        // Warps 2-5 read query half 0, warps 6-9 half 1: a warp may only read the TMEM
+        // lanes of its quarter (warp % 4), and each group covers all four quarters.
         const int quarter = warp & 3;                 // TMEM lanes 32*quarter .. +31
-        const int qrow = quarter * 32 + lane;         // query row inside a half
+        const int h = (warp - 2) >> 2;                // query half of this warp
+        const int qrow = quarter * 32 + lane;         // query row inside the half
         const int ethr = threadIdx.x - 64;            // scratch row of this epilogue thread
-        float best[2] = {-__int_as_float(0x7f800000), -__int_as_float(0x7f800000)};
-        int64_t best_row[2] = {-1, -1};
-        unsigned long long lst[2][LIST > 1 ? LIST : 1];
+        if (h < nhalf) {
+            float best = -__int_as_float(0x7f800000);
+            int64_t best_row = -1;
+            unsigned long long lst[LIST > 1 ? LIST : 1];
 #pragma unroll
-        for (int h = 0; h < 2; ++h)
-#pragma unroll
-            for (int j = 0; j < (LIST > 1 ? LIST : 1); ++j) lst[h][j] = 0ull;
-        int it = 0;
-        for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
-            const int acc = it % nbuf;
-            // one lane waits, the warp follows its verdict (tcgen05.ld needs the whole warp)
-            bool ok = true;
-            if (lane == 0) ok = wait_or_abort(&sm.acc_full[acc], static_cast<uint32_t>(it / nbuf) & 1u, sm);
-            ok = __shfl_sync(0xffffffffu, ok, 0);
-            if (!ok) break;
-            tc_fence_after();
-            const int64_t row0 = tile * kBN;
-            for (int h = 0; h < nhalf; ++h) {
+            for (int j = 0; j < (LIST > 1 ? LIST : 1); ++j) lst[j] = 0ull;
+            int it = 0;
+            for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
+                const int acc = it % nbuf;
+                // one lane waits, the warp follows its verdict (tcgen05.ld needs the whole warp)
+                bool ok = true;
+                if (lane == 0) ok = wait_or_abort(&sm.acc_full[acc], static_cast<uint32_t>(it / nbuf) & 1u, sm);
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                if (!ok) break;
+                tc_fence_after();
+                const int64_t row0 = tile * kBN;
 #pragma unroll 1
                 for (int c0 = 0; c0 < kBN; c0 += 32) {
                     float v[32];
@@ -261,7 +264,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         for (int j = 0; j < 32; ++j)
                             if (rbase + j < M) m = fmaxf(m, v[j]);
                     }
-                    if (m > best[h]) {
+                    if (m > best) {
                         // Slow path (rare per thread, but a warp takes it whenever one of
                         // its 32 queries does): mark the columns that beat the running
                         // best, park the scores in this thread's scratch row and visit
@@ -270,7 +273,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         uint32_t mask = 0u;
 #pragma unroll
                         for (int j = 0; j < 32; ++j) {
-                            const bool in = (full_cols || rbase + j < M) && v[j] > best[h];
+                            const bool in = (full_cols || rbase + j < M) && v[j] > best;
                             mask |= in ? (1u << j) : 0u;
                             sm.epi[ethr][j] = v[j];
                         }
@@ -278,38 +281,35 @@ __global__ void __launch_bounds__(kThreads, 1)
                             const int j = __ffs(static_cast<int>(mask)) - 1;
                             mask &= mask - 1u;
                             const float val = sm.epi[ethr][j];
-                            if (!(val > best[h])) continue;
+                            if (!(val > best)) continue;
                             if constexpr (LIST == 1) {
-                                best[h] = val;
-                                best_row[h] = rbase + j;
+                                best = val;
+                                best_row = rbase + j;
                             } else {
-                                // best[h] tracks the list's last score
-                                tc_list_insert<LIST>(lst[h], tc_key(val, rbase + j));
-                                if (lst[h][LIST - 1] != 0ull)
-                                    best[h] = unordered_tc(static_cast<uint32_t>(lst[h][LIST - 1] >> 32));
+                                // best tracks the list's last score
+                                tc_list_insert<LIST>(lst, tc_key(val, rbase + j));
+                                if (lst[LIST - 1] != 0ull)
+                                    best = unordered_tc(static_cast<uint32_t>(lst[LIST - 1] >> 32));
                             }
                         }
                     }
                 }
+                tc_fence_before();
+                mbar_arrive(&sm.acc_empty[acc]);
             }
-            tc_fence_before();
-            mbar_arrive(&sm.acc_empty[acc]);
-        }
-        __syncwarp();
-        for (int h = 0; h < nhalf; ++h) {
+            __syncwarp();
             const int q = h * kBM + qrow;
             if (LIST > 1 && q < nq) {
 #pragma unroll
                 for (int j = 0; j < kTopkStride; ++j)
                     partial[(static_cast<int64_t>(blockIdx.x) * n_queries + q0 + q) * kTopkStride + j] =
-                        j < LIST ? lst[h][j < LIST ? j : 0] : 0ull;
+                        j < LIST ? lst[j < LIST ? j : 0] : 0ull;
             }
             if (LIST == 1 && q < nq) {
                 unsigned long long key = 0ull;
-                if (best_row[h] >= 0)
-                    key = (static_cast<unsigned long long>(ordered_bits_tc(best[h])) << 32) |
-                          static_cast<unsigned long long>(0xffffffffu -
-                                                          static_cast<uint32_t>(best_row[h]));
+                if (best_row >= 0)
+                    key = (static_cast<unsigned long long>(ordered_bits_tc(best)) << 32) |
+                          static_cast<unsigned long long>(0xffffffffu - static_cast<uint32_t>(best_row));
                 partial[static_cast<int64_t>(blockIdx.x) * n_queries + q0 + q] = key;
             }
         }
