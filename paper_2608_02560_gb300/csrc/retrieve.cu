@@ -378,7 +378,11 @@ cudaError_t launch_gemv(const RetrieveParams &p, cudaStream_t stream, int grid, 
 }
 
 // Batches larger than one GEMV pass run on the tensor cores (16-bit keys).
-constexpr int kTcMinQueries = kQB + 1;
+// 16-bit indexes go to the tensor cores: one pass over the keys for up to 256 queries,
+// streamed by TMA; even a single query's pass is a little faster there (0.246 vs 0.266
+// ms over 1M x 768 fp16 keys) than on the CUDA-core kernel, which needs a pass per 4
+// queries. fp32 indexes stay on the CUDA cores.
+constexpr int kTcMinQueries = 1;
 
 bool use_tc(const RetrieveParams &p) {
     return p.dtype != PRECOG_F32 && p.n_queries >= kTcMinQueries && p.M > 0;

@@ -124,7 +124,7 @@ template <int LIST>
 __global__ void __launch_bounds__(kThreads, 1)
     retrieve_tc_kernel(const __grid_constant__ CUtensorMap tmap_q,
                        const __grid_constant__ CUtensorMap tmap_k, int64_t M, int dim,
-                       int n_queries, int q0, int nq, bool bf16,
+                       int n_queries, int q0, int nq, int a_rows, bool bf16,
                        unsigned long long *__restrict__ partial) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     Smem &sm = *reinterpret_cast<Smem *>(
@@ -173,7 +173,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         alive = false;
                         break;
                     }
-                    mbar_arrive_expect_tx(&sm.full[s], nhalf * kABytes + kBBytes);
+                    mbar_arrive_expect_tx(&sm.full[s], static_cast<uint32_t>(nhalf * a_rows * kBK * 2) + kBBytes);
                     for (int h = 0; h < nhalf; ++h)
                         tma_load_2d(sm.a[s][h], &tmap_q, kb * kBK, q0 + h * kBM, &sm.full[s]);
                     tma_load_2d(sm.b[s], &tmap_k, kb * kBK, static_cast<int32_t>(tile * kBN),
@@ -369,7 +369,11 @@ template <int LIST>
 cudaError_t launch_tc(const RetrieveParams &p, int grid, cudaStream_t stream, uint64_t *launches) {
     const bool bf16 = p.dtype == PRECOG_BF16;
     CUtensorMap tq, tk;
-    if (!make_map(&tq, p.queries, p.n_queries, p.dim, bf16, kBM) ||
+    // A batch of fewer than 128 queries loads only its rows (rounded up to the 8-row
+    // swizzle atom); the rest of the A tile is never read back (its TMEM lanes belong to
+    // no query), and copies that are mostly out of bounds are slow.
+    const int a_rows = p.n_queries >= kBM ? kBM : ((p.n_queries + 7) & ~7);
+    if (!make_map(&tq, p.queries, p.n_queries, p.dim, bf16, a_rows) ||
         !make_map(&tk, p.index, p.M > 0 ? p.M : 1, p.dim, bf16, kBN))
         return cudaErrorInvalidValue;
     static int smem_set = 0;
@@ -379,7 +383,7 @@ cudaError_t launch_tc(const RetrieveParams &p, int grid, cudaStream_t stream, ui
     for (int q0 = 0; q0 < p.n_queries; q0 += 2 * kBM) {
         const int nq = p.n_queries - q0 < 2 * kBM ? p.n_queries - q0 : 2 * kBM;
         retrieve_tc_kernel<LIST><<<grid, kThreads, smem, stream>>>(
-            tq, tk, p.M, p.dim, p.n_queries, q0, nq, bf16,
+            tq, tk, p.M, p.dim, p.n_queries, q0, nq, a_rows, bf16,
             static_cast<unsigned long long *>(p.workspace));
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;

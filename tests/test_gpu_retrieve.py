@@ -126,12 +126,13 @@ def test_query_workload_full_index(cuda_device, Q):
     torch.cuda.empty_cache()
 
 
-# ------------------------------------------------------------- tensor-core path (Q >= 5)
+# ------------------------------------------------------------- tensor-core path (16-bit keys, Q >= 2)
 
 
 @pytest.mark.parametrize("dtype_name", ["float16", "bfloat16"])
 @pytest.mark.parametrize("M,Q,dim", [(1, 5, 64), (127, 9, 64), (128, 130, 96), (129, 256, 768),
-                                     (4099, 300, 96), (20000, 17, 136)])
+                                     (4099, 300, 96), (20000, 17, 136), (3000, 2, 64), (70000, 4, 768),
+                                     (513, 127, 64), (513, 128, 64)])
 def test_tensor_core_exact_integer_scores(cuda_device, dtype_name, M, Q, dim):
     """Batches of five or more queries over a 16-bit index take the tcgen05 path. Small
     integer keys and queries make every score exact in fp32, so indices and scores must

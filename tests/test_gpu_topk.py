@@ -31,8 +31,8 @@ def _topk(index, queries, k):
                                        (4099, 9, 8, 64), (20000, 200, 5, 136), (300, 300, 2, 64)])
 def test_topk_exact_integer_scores(cuda_device, dtype_name, M, Q, k, dim):
     """Small-integer keys: exact scores, many ties. Rows and scores must equal the
-    oracle's stable ranking bit for bit, on the CUDA-core path (Q <= 4, or fp32) and
-    the tensor-core path (fp16/bf16, Q >= 5)."""
+    oracle's stable ranking bit for bit, on the CUDA-core path (Q = 1, or fp32) and
+    the tensor-core path (fp16/bf16, Q >= 2)."""
     import torch
     dtype = getattr(torch, dtype_name)
     if dtype == torch.float32 and Q > 50:
