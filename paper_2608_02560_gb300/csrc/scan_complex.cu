@@ -26,13 +26,29 @@ constexpr float kInv2Pi = 0.15915494309189535f;
 constexpr float k2PiHi = 6.28318548202514648f;     // fp32 nearest to 2*pi
 constexpr float k2PiLo = -1.7484556000744487e-07f; // 2*pi - k2PiHi
 
-__device__ __forceinline__ void sincos_reduced(float hi, float lo, float &s, float &c) {
-    const float k = rintf(hi * kInv2Pi);
-    float r = fmaf(-k, k2PiHi, hi);
-    r = fmaf(-k, k2PiLo, r);
-    r += lo;
-    asm("sin.approx.ftz.f32 %0, %1;" : "=f"(s) : "f"(r));
-    asm("cos.approx.ftz.f32 %0, %1;" : "=f"(c) : "f"(r));
+// sin and cos of the phases (th + tl) of two state indices at once. th is the rounded
+// product dt * A_im and tl its exact error (an fma), so th + tl is the phase to twice
+// fp32 precision; it is reduced by k = rint(th / 2pi) with 2pi split into a float and
+// its remainder (Cody-Waite) before the SFU sine and cosine. Packed fp32x2 arithmetic
+// halves the issue slots; each lane rounds exactly as the scalar sequence would.
+__device__ __forceinline__ void sincos_pair(f2 th, f2 tl, f2 &s, f2 &c) {
+    // k = rint(th / 2pi) on the FMA pipe: adding 1.5 * 2^23 rounds to an integer (round to
+    // nearest even) for |th / 2pi| < 2^22; subtracting it again is exact. This keeps the
+    // rounding off the SFU/conversion pipe, which the exponential, sine and cosine fill.
+    const f2 big = pack2(12582912.f, 12582912.f), nbig = pack2(-12582912.f, -12582912.f);
+    const f2 one = pack2(1.f, 1.f);
+    const f2 k = fma2(fma2(th, pack2(kInv2Pi, kInv2Pi), big), one, nbig);
+    f2 r = fma2(k, pack2(-k2PiHi, -k2PiHi), th);
+    r = fma2(k, pack2(-k2PiLo, -k2PiLo), r);
+    r = fma2(r, one, tl);
+    float r0, r1, s0, s1, c0, c1;
+    unpack2(r, r0, r1);
+    asm("sin.approx.ftz.f32 %0, %1;" : "=f"(s0) : "f"(r0));
+    asm("cos.approx.ftz.f32 %0, %1;" : "=f"(c0) : "f"(r0));
+    asm("sin.approx.ftz.f32 %0, %1;" : "=f"(s1) : "f"(r1));
+    asm("cos.approx.ftz.f32 %0, %1;" : "=f"(c1) : "f"(r1));
+    s = pack2(s0, s1);
+    c = pack2(c0, c1);
 }
 
 // One 16-value B or C row (32 or 64 bytes, 16-byte aligned), fetched raw with
@@ -94,12 +110,19 @@ __global__ void __launch_bounds__(kBlock)
     const TIn *Cl = HAS_Y ? static_cast<const TIn *>(p.C) + layer * p.ls_bc : nullptr;
     const float2 *Al = reinterpret_cast<const float2 *>(p.A) + (static_cast<int64_t>(layer) * D + d) * kN;
 
-    float ar[kN], ai[kN], hr[kN], hi[kN];
+    // state indices in pairs (2i, 2i+1): A_re * log2 e, A_im, -A_im, and the state
+    constexpr int kP = kN / 2;
+    f2 ar[kP], ai[kP], nai[kP];
+    float hr[kN], hi[kN];
+#pragma unroll
+    for (int i = 0; i < kP; ++i) {
+        const float2 a0 = Al[2 * i], a1 = Al[2 * i + 1];
+        ar[i] = pack2(a0.x * kLog2e, a1.x * kLog2e);
+        ai[i] = pack2(a0.y, a1.y);
+        nai[i] = pack2(-a0.y, -a1.y);
+    }
 #pragma unroll
     for (int n = 0; n < kN; ++n) {
-        const float2 a = Al[n];
-        ar[n] = a.x * kLog2e;
-        ai[n] = a.y;
         hr[n] = 0.f;
         hi[n] = 0.f;
     }
@@ -146,21 +169,29 @@ __global__ void __launch_bounds__(kBlock)
             nb.load(Bl + (t + 1) * kN);
             if constexpr (HAS_Y) nc.load(Cl + (t + 1) * kN);
         }
-        float y = 0.f;
+        const f2 dd = pack2(dv, dv), uu = pack2(u, u);
+        f2 y2 = pack2(0.f, 0.f);
 #pragma unroll
-        for (int n = 0; n < kN; ++n) {
-            const float mag = ex2(dv * ar[n]);
-            const float th = dv * ai[n];
-            const float tl = fmaf(dv, ai[n], -th);   // exact error of the product
-            float s, c;
-            sincos_reduced(th, tl, s, c);
-            const float are = mag * c, aim = mag * s;
-            const float nr = fmaf(are, hr[n], fmaf(-aim, hi[n], u * b[n]));
-            const float ni = fmaf(are, hi[n], aim * hr[n]);
-            hr[n] = nr;
-            hi[n] = ni;
-            if constexpr (HAS_Y) y = fmaf(cr[n], nr, y);
+        for (int i = 0; i < kP; ++i) {
+            float e0, e1;
+            unpack2(mul2(dd, ar[i]), e0, e1);
+            const f2 mag = pack2(ex2(e0), ex2(e1));
+            const f2 th = mul2(dd, ai[i]);
+            const f2 tl = fma2(dd, ai[i], mul2(dd, nai[i]));   // exact error of the product
+            f2 sn, cs;
+            sincos_pair(th, tl, sn, cs);
+            const f2 are = mul2(mag, cs), aim = mul2(mag, sn);
+            const f2 h_r = pack2(hr[2 * i], hr[2 * i + 1]), h_i = pack2(hi[2 * i], hi[2 * i + 1]);
+            const f2 nh_i = pack2(-hi[2 * i], -hi[2 * i + 1]);
+            const f2 nr = fma2(are, h_r, fma2(aim, nh_i, mul2(uu, pack2(b[2 * i], b[2 * i + 1]))));
+            const f2 ni = fma2(are, h_i, mul2(aim, h_r));
+            unpack2(nr, hr[2 * i], hr[2 * i + 1]);
+            unpack2(ni, hi[2 * i], hi[2 * i + 1]);
+            if constexpr (HAS_Y) y2 = fma2(pack2(cr[2 * i], cr[2 * i + 1]), nr, y2);
         }
+        float y0, y1;
+        unpack2(y2, y0, y1);
+        const float y = y0 + y1;
         if constexpr (HAS_Y) {
             const int64_t yo = (static_cast<int64_t>(layer) * p.T_tot + t) * D + d;
             if (p.y_dtype == PRECOG_F32) static_cast<float *>(p.y)[yo] = y;
