@@ -4,18 +4,18 @@
 One step = one pass of the whole hot path over one batch of synthetic input:
   * corpus encode of the paper-shaped workload: 24 independent layers (D=256,
     N=16), 4096 chunks x 3000 tokens, bf16 inputs, fp32 state, captured into a
-    bf16 bank of 192 KB per chunk (24 C-ABI encode calls, one per layer);
+    bf16 bank of 192 KB per chunk (C-ABI encode calls of S layers each);
   * the query-time path: top-1 retrieval of a query batch over 1,000,000
     unit-norm fp16 keys of dim 768, injection of the retrieved 192 KB state from
     a 1,000,000-entry bank and scan prefill of 64 query tokens per query.
 
 value = corpus tokens encoded per second (through all 24 layers) by all ranks.
 The 24 layers' inputs (12.98 GB each, 311 GB in all) exceed HBM: `--input-sets`
-independently generated layer inputs stay resident and layer l reads set
-l mod S. Every encode call still streams its full 12.98 GB from HBM (far above
-the 129 MB L2), so the timed traffic and work equal those of 24 independent
-layers; generating the synthetic inputs is not part of the method and is
-timed separately. The retrieve+inject+prefill p50 latency is measured after the
+S (default 4) independently generated layer inputs stay resident, contiguous,
+and one encode call covers S layers, layer l reading set l mod S. Every layer
+still streams its full 12.98 GB from HBM (far above the 129 MB L2), so the timed
+traffic and work equal those of 24 independent layers; generating the synthetic
+inputs is not part of the method and is timed separately. The retrieve+inject+prefill p50 latency is measured after the
 timed steps, per query batch, with an L2 flush before every iteration.
 
 `--impl reference` times the CPU oracle (fp64, sequential) on a bounded sample
@@ -52,7 +52,9 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--input-sets", type=int, default=2)
+    ap.add_argument("--input-sets", type=int, default=4,
+                    help="independent layer inputs kept resident; each encode call covers this many "
+                         "layers (must divide 24)")
     ap.add_argument("--query-batch", type=int, default=1)
     ap.add_argument("--latency-iters", type=int, default=200)
     ap.add_argument("--e2e-steps", type=int, default=2)
@@ -86,8 +88,8 @@ def peaks():
 
 
 def profiled_traffic():
-    """Per-launch DRAM traffic from the committed ncu summary, if it was taken on the
-    current scan kernel source (else None)."""
+    """DRAM traffic of one single-layer encode launch from the committed ncu summary, if
+    it was taken on the current scan kernel source (else None)."""
     if not os.path.exists(PROFILE):
         return None
     text = open(PROFILE).read()
@@ -450,13 +452,25 @@ def main():
     T = int(off_np[-1])
     off = torch.from_numpy(off_np).to(dev)
 
+    # S independently drawn layer inputs, contiguous so that one C-ABI call encodes S
+    # layers (S x 4096 CTAs: fewer partial last waves than one layer per launch)
+    S = args.input_sets
+    if S < 1 or L % S:
+        raise SystemExit(f"--input-sets must divide {L}")
     t_gen = time.perf_counter()
-    sets = [synth.device_scan_inputs(T, D, N, seed, s, dev, with_C=False)
-            for s in range(args.input_sets)]
+    x_all = torch.empty((S, T, D), dtype=torch.bfloat16, device=dev)
+    dt_all = torch.empty_like(x_all)
+    B_all = torch.empty((S, T, N), dtype=torch.bfloat16, device=dev)
+    sets = [synth.device_scan_inputs(T, D, N, seed, s, dev, with_C=False,
+                                     out={"x": x_all[s], "dt": dt_all[s], "B": B_all[s]})
+            for s in range(S)]
     torch.cuda.synchronize()
-    gen_s_per_layer = (time.perf_counter() - t_gen) / args.input_sets
+    gen_s_per_layer = (time.perf_counter() - t_gen) / S
     bank = torch.empty((shape.n_chunks, L, D, N), dtype=torch.bfloat16, device=dev)
-    scan_in = [pg.scan_inputs(s["x"], s["dt"], s["B"], s["A"], a_kind=pg.PRECOG_A_POWER) for s in sets]
+    A_all = torch.stack([st["A"] for st in sets]).contiguous()
+    call_in = pg.scan_inputs(x_all, dt_all, B_all, A_all, a_kind=pg.PRECOG_A_POWER)
+    scan_in = [pg.scan_inputs(st["x"], st["dt"], st["B"], st["A"], a_kind=pg.PRECOG_A_POWER) for st in sets]
+    calls = L // S
 
     # query-time workload
     M, dim, Tq, Q = synth.QUERY_INDEX_M, synth.QUERY_DIM, synth.QUERY_TOKENS, args.query_batch
@@ -486,16 +500,16 @@ def main():
                                      state_out=b["h"], stream=stream)
 
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-          for _ in range(L * args.steps)]
+          for _ in range(calls * args.steps)]
 
     def step(k=None):
-        for l in range(L):
+        # layers c*S .. c*S+S-1 in one call; layer l reads input set l mod S
+        for c in range(calls):
             if k is not None:
-                ev[k * L + l][0].record()
-            pg.precog_encode_chunks(scan_in[l % args.input_sets], off, T, states_out=bank,
-                                    layer0=l, L_total=L)
+                ev[k * calls + c][0].record()
+            pg.precog_encode_chunks(call_in, off, T, states_out=bank, layer0=c * S, L_total=L)
             if k is not None:
-                ev[k * L + l][1].record()
+                ev[k * calls + c][1].record()
         query_path(qb)
 
     for _ in range(args.warmup):
@@ -527,11 +541,13 @@ def main():
     ms_per_step = elapsed_ms / args.steps
 
     hbm, peak_src = peaks()
-    bpl = scan_bytes_per_launch(T, shape.n_chunks, D, N)
+    bpl = S * scan_bytes_per_launch(T, shape.n_chunks, D, N)
     avg_scan_ms = statistics.mean(scan_ms)
     achieved = bpl / (avg_scan_ms * 1e-3) / 1e9
+    layer_traffic = profiled_traffic()
     roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                "frac": achieved / hbm, "traffic": profiled_traffic(),
+                "frac": achieved / hbm, "traffic": None if layer_traffic is None else S * layer_traffic,
+                "layers_per_launch": S,
                 "kernel": "scan_kernel (encode, capture)", "peak_source": peak_src,
                 "algorithmic_bytes_per_launch": bpl, "avg_launch_ms": avg_scan_ms}
 
@@ -553,7 +569,6 @@ def main():
                     for k in ("idx", "score", "y", "h")}
         copy_stream = torch.cuda.Stream(device=dev)
         comp = torch.cuda.current_stream(dev)
-        S = args.input_sets
         h2d = sum(host[k].numel() * host[k].element_size() for k in host) * L
         h2d += sum(hq[k].numel() * hq[k].element_size() for k in hq)
         d2h = bank.numel() * bank.element_size()
@@ -662,7 +677,7 @@ def main():
                 "config": {"workload": "paper-shaped corpus encode + query-time path",
                            "layers": L, "D": D, "N": N, "chunks": shape.n_chunks,
                            "chunk_tokens": shape.chunk_len, "state_bytes_per_chunk": L * D * N * 2,
-                           "input_sets_resident": args.input_sets,
+                           "input_sets_resident": S, "layers_per_encode_call": S,
                            "index_rows": M, "index_dim": dim, "bank_entries": M,
                            "query_batch": Q, "query_tokens": Tq, "parallelism": f"dp{world}",
                            "l2": "inputs larger than L2 (12.98 GB per layer, 1.5 GB index)"},

@@ -310,6 +310,37 @@ def _sampled_check(dev, shape, layer, sample_chunks, y_mode=False, seed=0):
     return worst
 
 
+def test_paper_shaped_multi_layer_call_sampled(cuda_device):
+    """The launch the benchmark times: one call encodes 4 paper-shaped layers (4096 chunks x
+    3000 tokens each, contiguous inputs of 4 independent draws) into layers 8..11 of the
+    24-layer bf16 bank; sampled chunks of every layer vs the oracle, other layers untouched."""
+    import torch
+    pg = _pg()
+    d = cuda_device
+    shape, S, layer0 = synth.PAPER, 4, 8
+    off_np = synth.shape_offsets(shape, 0)
+    T = int(off_np[-1])
+    x = torch.empty((S, T, shape.D), dtype=torch.bfloat16, device=d)
+    dt = torch.empty_like(x)
+    B = torch.empty((S, T, shape.N), dtype=torch.bfloat16, device=d)
+    sets = [synth.device_scan_inputs(T, shape.D, shape.N, 0, l, d, with_C=False,
+                                     out={"x": x[l], "dt": dt[l], "B": B[l]}) for l in range(S)]
+    A = torch.stack([st["A"] for st in sets]).contiguous()
+    states = torch.full((shape.n_chunks, shape.n_layers, shape.D, shape.N), 5.0, dtype=torch.bfloat16,
+                        device=d)
+    pg.precog_encode_chunks(pg.scan_inputs(x, dt, B, A, a_kind=pg.PRECOG_A_POWER),
+                            torch.from_numpy(off_np).to(d), T, states_out=states, layer0=layer0,
+                            L_total=shape.n_layers)
+    assert pg.precog_device_status()[0] == 0
+    assert bool(torch.all(states[:, :layer0] == 5.0)) and bool(torch.all(states[:, layer0 + S:] == 5.0))
+    An = sets[0]["A"].cpu().numpy()
+    for l in range(S):
+        for c in (0, 2047, shape.n_chunks - 1):
+            sl = slice(int(off_np[c]), int(off_np[c + 1]))
+            ref_h, _ = oracle.rollout(to_np(x[l, sl]), to_np(dt[l, sl]), An, to_np(B[l, sl]))
+            assert rel_err_stored(to_np(states[c, layer0 + l]), ref_h) < TOL_BF16, (l, c)
+
+
 def test_wide_single_layer_full_size(cuda_device):
     """1 layer, D=2048, N=16, 1024 chunks x 512 tokens, bf16 (capture and y modes)."""
     _sampled_check(cuda_device, synth.WIDE, 0, [0, 511, 1023])
