@@ -48,6 +48,9 @@ struct ScanParams {
     const int64_t *traj_offsets;  // [n_chunks+1] first entry of each chunk
 };
 
+// SM count of the current device (cached per device; 1 if it cannot be read).
+int device_sm_count();
+
 // cuTensorMapEncodeTiled through the runtime's driver entry point (no link against
 // libcuda); false if the entry point is missing or the driver rejects the map.
 bool encode_tiled_map(CUtensorMap *map, CUtensorMapDataType dtype, cuuint32_t rank, const void *base,

@@ -323,16 +323,7 @@ __global__ void finalize_topk_kernel(const unsigned long long *__restrict__ part
     }
 }
 
-int num_sms() {
-    static int sms = 0;
-    if (sms == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        if (sms <= 0) sms = 1;
-    }
-    return sms;
-}
+int num_sms() { return device_sm_count(); }
 
 constexpr int kRowsPerWarpPass = 4;
 

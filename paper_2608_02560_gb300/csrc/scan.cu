@@ -742,15 +742,7 @@ int pick_slice(int D, int sz, int cpt) {
 
 // True when a full-width launch would have fewer CTAs than the device has SMs.
 bool few_items(const ScanParams &p) {
-    static int sms = 0;
-    if (sms == 0) {
-        int dev = 0, n = 0;
-        if (cudaGetDevice(&dev) == cudaSuccess &&
-            cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && n > 0)
-            sms = n;
-        else
-            return false;
-    }
+    const int sms = device_sm_count();
     const int64_t slices = (p.D + kMaxSlice - 1) / kMaxSlice;
     return static_cast<int64_t>(p.n_layers) * p.n_chunks * slices < sms;
 }
