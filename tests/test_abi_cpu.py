@@ -125,3 +125,27 @@ def test_retrieve_rejects_bad_arguments(lib):
     assert f(FAKE, 2, 100, 768, None, 1, FAKE, FAKE, FAKE, 1 << 20, None) == 1
     assert f(FAKE, 2, 100, 768, FAKE, 0, FAKE, FAKE, FAKE, 0, None) == 0       # no queries
     assert lib.precog_retrieve_workspace_size(100, 768, 4) >= 4 * 8
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    """No CPU fallback: loading the binding against a path with no libprecog.so raises
+    instead of computing anything another way."""
+    import paper_2608_02560_gb300 as pg
+    saved = pg._lib
+    try:
+        pg._lib = None
+        with pytest.raises(ImportError):
+            pg.load_library(str(tmp_path / "libprecog.so"))
+    finally:
+        pg._lib = saved
+
+
+def test_product_package_does_not_import_the_oracle():
+    """The product path never reaches the test oracle: no module of the package names it."""
+    pkg = os.path.join(ROOT, "paper_2608_02560_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h", ".cpp")):
+                text = open(os.path.join(dirpath, f)).read()
+                assert not re.search(r"^\s*(import|from)\s+oracle\b", text, flags=re.M), f
+                assert "precog_oracle" not in text, f
