@@ -64,7 +64,8 @@ def parse_args():
     ap.add_argument("--no-extras", action="store_true",
                     help="skip the measurements of the extension rows (top-k, trajectory, complex A, SMC)")
     ap.add_argument("--case", choices=["full", "scan-small", "retrieve-small", "topk-small", "prefill-small",
-                                       "wide-encode", "wide-encode-y", "ragged-encode"],
+                                       "wide-encode", "wide-encode-y", "ragged-encode", "trajectory-small",
+                                       "complex-small", "consolidate"],
                     default="full",
                     help="small single-kernel cases (a few GB) used for profiler captures")
     return ap.parse_args()
@@ -250,6 +251,37 @@ def run_case(args):
         fn = lambda: pg.precog_encode_chunks(si, off, T, states_out=bank, layer0=0, L_total=shape.n_layers)
         res["algorithmic_bytes_per_launch"] = scan_bytes_per_launch(T, chunks, shape.D, shape.N)
         res["scale_to_full_launch"] = shape.n_chunks * shape.chunk_len / T
+    elif args.case in ("trajectory-small", "complex-small"):
+        # the scan-small rows (3040 chunks x 1000 tokens, D=256): every 250th state kept, or
+        # the complex diagonal A of Eq. 1 (real part -(n+1), imaginary part pi*n)
+        shape, chunks, clen = synth.PAPER, 3040, 1000
+        off_np = synth.fixed_offsets(chunks, clen)
+        T = int(off_np[-1])
+        inp = synth.device_scan_inputs(T, shape.D, shape.N, 0, 0, dev, with_C=False)
+        off = torch.from_numpy(off_np).to(dev)
+        in_bytes = T * (2 * shape.D + shape.N) * 2
+        if args.case == "trajectory-small":
+            stride = 250
+            eo = torch.arange(chunks + 1, dtype=torch.int64, device=dev) * (clen // stride)
+            traj = torch.empty((chunks * (clen // stride), 1, shape.D, shape.N), dtype=torch.bfloat16, device=dev)
+            si = pg.scan_inputs(inp["x"], inp["dt"], inp["B"], inp["A"], a_kind=pg.PRECOG_A_POWER)
+            fn = lambda: pg.precog_encode_trajectory(si, off, T, stride, eo, traj)
+            res["algorithmic_bytes_per_launch"] = in_bytes + traj.numel() * 2
+        else:
+            im = (math.pi * torch.arange(shape.N, device=dev, dtype=torch.float32)).expand(shape.D, shape.N)
+            A = torch.complex(inp["A"], im).contiguous()
+            cst = torch.empty((chunks, 1, shape.D, shape.N, 2), dtype=torch.bfloat16, device=dev)
+            si = pg.scan_inputs(inp["x"], inp["dt"], inp["B"], A, a_kind=pg.PRECOG_A_COMPLEX)
+            fn = lambda: pg.precog_encode_chunks(si, off, T, states_out=cst)
+            res["algorithmic_bytes_per_launch"] = in_bytes + cst.numel() * 2
+    elif args.case == "consolidate":
+        # 4096 24-layer bf16 states (805 MB) folded into 64 semantic slots
+        n, elems = 4096, 24 * 256 * 16
+        states = synth.device_normal_bank(n, elems, 22, dev)
+        slots = torch.arange(n, dtype=torch.int64, device=dev) * 7 % 64
+        sem = torch.zeros((64, elems), dtype=torch.float32, device=dev)
+        fn = lambda: pg.precog_smc_consolidate(sem, states, slots, 0.1)
+        res["algorithmic_bytes_per_launch"] = n * elems * 2 + 2 * sem.numel() * 4
     elif args.case in ("wide-encode", "wide-encode-y", "ragged-encode"):
         # one layer of the single-layer wide encode (D=2048, 1024 x 512 tokens; capture or
         # readout) or of the ragged encode (D=512, 8192 chunks of 256..4096 tokens)
@@ -300,7 +332,7 @@ def run_case(args):
         ev[2 * i + 1].record()
     torch.cuda.synchronize()
     res["ms"] = [ev[2 * i].elapsed_time(ev[2 * i + 1]) for i in range(3)]
-    if args.case in ("wide-encode", "wide-encode-y", "ragged-encode"):
+    if "algorithmic_bytes_per_launch" in res:
         best = min(res["ms"][1:])
         res["achieved_gbs"] = res["algorithmic_bytes_per_launch"] / (best * 1e-3) / 1e9
         res["frac_hbm"] = res["achieved_gbs"] / peaks()[0]
