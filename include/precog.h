@@ -322,6 +322,19 @@ precog_status precog_smc_consolidate(float *semantic, int64_t n_slots, int64_t s
                                      int64_t n, float alpha, void *stream);
 
 /*
+ * precog_selftest_wait_timeout -- diagnostic; the paper has no counterpart.
+ * Every kernel here that waits on copies (TMA completion on an mbarrier) gives
+ * the wait an iteration limit: when it runs out, the kernel sets
+ * PRECOG_DEV_TIMEOUT in its device status word and returns, so a lost copy
+ * becomes an error status instead of a hung GPU. This call exercises that path
+ * on purpose: one warp waits, for `iterations` try-wait rounds (1 .. 2^20), on
+ * an mbarrier that nothing arrives on, records PRECOG_DEV_TIMEOUT and returns.
+ * The next precog_device_status on the stream reports PRECOG_ERR_TIMEOUT with
+ * that bit (and clears it); the context stays usable. Asynchronous on `stream`.
+ */
+precog_status precog_selftest_wait_timeout(uint32_t iterations, void *stream);
+
+/*
  * precog_device_status -- synchronise `stream`, then report and clear the
  * device status word shared by all calls on this device. *bits_out receives
  * the PRECOG_DEV_* bits seen since the last clear. Returns PRECOG_OK when no

@@ -86,6 +86,8 @@ def load_library(path: str = LIB_PATH):
     lib.precog_prefill_composed.restype = i32
     lib.precog_prefill_composed.argtypes = [ctypes.POINTER(ScanInputs), i32, i32, vp, i32, i64, i32,
                                             i32, i32, vp, vp, ctypes.c_float, vp, i32, vp, i32, vp]
+    lib.precog_selftest_wait_timeout.restype = i32
+    lib.precog_selftest_wait_timeout.argtypes = [ctypes.c_uint32, vp]
     lib.precog_device_status.restype = i32
     lib.precog_device_status.argtypes = [vp, ctypes.POINTER(ctypes.c_uint32)]
     lib.precog_status_string.restype = ctypes.c_char_p
@@ -278,6 +280,12 @@ def precog_smc_consolidate(semantic, states, slots, alpha: float, stream=None):
     _check(lib.precog_smc_consolidate(
         _ptr(semantic), n_slots, elems, _ptr(states), _dtype_code(states), _ptr(slots),
         states.shape[0], alpha, _stream(stream)))
+
+
+def precog_selftest_wait_timeout(iterations: int = 4096, stream=None):
+    """Run the bounded-wait failure path on purpose (a wait that nothing completes): the
+    next precog_device_status reports PRECOG_ERR_TIMEOUT. Diagnostic only."""
+    _check(load_library().precog_selftest_wait_timeout(iterations, _stream(stream)))
 
 
 def precog_device_status(stream=None):

@@ -428,6 +428,14 @@ precog_status precog_smc_consolidate(float *semantic, int64_t n_slots, int64_t s
     return ok();
 }
 
+precog_status precog_selftest_wait_timeout(uint32_t iterations, void *stream) {
+    if (iterations < 1 || iterations > (1u << 20))
+        return fail(PRECOG_ERR_INVALID_ARG, "iterations must be in [1, 2^20]");
+    cudaError_t e = precog::launch_wait_timeout(iterations, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "self-test launch");
+    return ok();
+}
+
 precog_status precog_device_status(void *stream, uint32_t *bits_out) {
     if (bits_out == nullptr) return fail(PRECOG_ERR_INVALID_ARG, "bits_out is NULL");
     *bits_out = 0;
@@ -443,7 +451,10 @@ precog_status precog_device_status(void *stream, uint32_t *bits_out) {
     if (e != cudaSuccess) return cuda_fail(e, "read smc status");
     e = precog::scan_complex_status_word_read_clear(&z);
     if (e != cudaSuccess) return cuda_fail(e, "read complex scan status");
-    *bits_out = a | b | c | z;
+    uint32_t w = 0;
+    e = precog::selftest_status_word_read_clear(&w);
+    if (e != cudaSuccess) return cuda_fail(e, "read self-test status");
+    *bits_out = a | b | c | z | w;
     if (*bits_out == 0) return ok();
     if (*bits_out & PRECOG_DEV_TIMEOUT)
         return fail(PRECOG_ERR_TIMEOUT, "a device-side wait gave up (bits 0x%x)", *bits_out);

@@ -48,6 +48,10 @@ struct ScanParams {
     const int64_t *traj_offsets;  // [n_chunks+1] first entry of each chunk
 };
 
+// Bounded-wait self-test (selftest.cu).
+cudaError_t launch_wait_timeout(uint32_t limit, cudaStream_t stream);
+cudaError_t selftest_status_word_read_clear(uint32_t *bits);
+
 // SM count of the current device (cached per device; 1 if it cannot be read).
 int device_sm_count();
 

@@ -149,3 +149,10 @@ def test_product_package_does_not_import_the_oracle():
                 text = open(os.path.join(dirpath, f)).read()
                 assert not re.search(r"^\s*(import|from)\s+oracle\b", text, flags=re.M), f
                 assert "precog_oracle" not in text, f
+
+
+def test_selftest_rejects_bad_iteration_counts(lib):
+    lib.precog_selftest_wait_timeout.argtypes = [ctypes.c_uint32, ctypes.c_void_p]
+    lib.precog_selftest_wait_timeout.restype = ctypes.c_int32
+    assert lib.precog_selftest_wait_timeout(0, None) == 1
+    assert lib.precog_selftest_wait_timeout((1 << 20) + 1, None) == 1
