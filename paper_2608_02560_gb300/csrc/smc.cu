@@ -106,11 +106,10 @@ __device__ __forceinline__ void describe_batch(BatchMeta &m, int64_t raw, int64_
     int64_t sl = INT64_MIN;                       // lanes beyond the batch never match
     if (lane < kU) {
         sl = raw;
-        if (sl >= n_slots) {
+        if (sl >= n_slots || sl < -1) {
             atomicOr(&g_smc_status, PRECOG_DEV_BAD_INDEX);
             sl = -1;
         }
-        if (sl < -1) sl = -1;
     }
     const bool valid = lane < kU && sl >= 0;
     const uint32_t same = __match_any_sync(0xffffffffu, sl);
@@ -283,7 +282,7 @@ __global__ void __launch_bounds__(kSlotThreads)
         for (int r = 0; r < 4; ++r) {
             const int64_t c = c0 + r * kSlotThreads + tid;
             sl[r] = c < n ? slots[c] : -1;
-            if (flagger && sl[r] >= n_slots) atomicOr(&g_smc_status, PRECOG_DEV_BAD_INDEX);
+            if (flagger && (sl[r] >= n_slots || sl[r] < -1)) atomicOr(&g_smc_status, PRECOG_DEV_BAD_INDEX);
         }
         if (tid == 0) s_total = 0;
         __syncthreads();
@@ -331,6 +330,260 @@ __global__ void __launch_bounds__(kSlotThreads)
         if (e[i] < elems) store_sem<VEC>(sem + slot * elems + e[i], v[i]);
 }
 
+// The per-slot fold with the states streamed through shared memory by the TMA
+// engine. A persistent CTA takes a contiguous run of (slot, element range)
+// tiles. Its producer warp streams the slot ids through a ring of kIdRing
+// chunks of kIdChunk ids (bulk copies kIdRing chunks ahead, so that finding
+// the deposits does not wait on one round trip per chunk), matches them in
+// deposit order and, for each deposit of the tile's slot, queues one bulk copy
+// of that deposit's range of elements into a ring of kRing stages; the
+// kBulkConsumers consumer threads fold every stage into the range's semantic
+// values, which stay in registers for the whole tile. A stage tagged
+// kTagTileEnd carries no data and closes the tile: its values are stored and
+// the next tile's loaded while the ring keeps streaming. Each state element
+// crosses HBM once, each semantic element is read and written once.
+constexpr int kBulkConsumers = 256;
+constexpr int kBulkThreads = kBulkConsumers + 32;
+constexpr int kStageBytes = 16384;
+constexpr int kRing = 6;
+constexpr int kChunksPerThread = kStageBytes / 16 / kBulkConsumers;
+constexpr int kIdChunk = 256;
+constexpr int kIdRing = 6;
+constexpr int32_t kTagData = 1;
+constexpr int32_t kTagTileEnd = 2;
+static_assert(kChunksPerThread * 16 * kBulkConsumers == kStageBytes, "stage = whole 16-byte chunks");
+static_assert(kIdChunk % 32 == 0, "whole warps of ids");
+
+struct BulkSmem {
+    unsigned char ring[kRing][kStageBytes];
+    int64_t ids[kIdRing][kIdChunk];
+    uint64_t full[kRing];
+    uint64_t empty[kRing];
+    uint64_t idfull[kIdRing];
+    int32_t tag[kRing];
+    int32_t abort;
+};
+
+// Bounded wait that also gives up once another role of the CTA has given up.
+__device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, const volatile int32_t *abort) {
+    for (uint32_t i = 0; i < kWaitLimit; ++i) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((i & 255u) == 255u && *abort) return false;
+    }
+    return false;
+}
+
+// Producer: claim stage g (wait until the consumers released its previous
+// use), tag it and start its copy (src == nullptr: a tile-end marker).
+// Warp-uniform result; false when the wait ran out or the CTA gave up.
+__device__ __forceinline__ bool produce_stage(BulkSmem &sm, uint32_t g, int lane, const void *src,
+                                              uint32_t bytes) {
+    const int s = static_cast<int>(g % kRing);
+    int ok = 1;
+    if (lane == 0) {
+        ok = wait_or_abort(&sm.empty[s], ((g / kRing) & 1u) ^ 1u, &sm.abort);
+        if (ok) {
+            sm.tag[s] = src ? kTagData : kTagTileEnd;
+            if (src) {
+                mbar_arrive_expect_tx(&sm.full[s], bytes);
+                bulk_g2s(sm.ring[s], src, bytes, &sm.full[s]);
+            } else {
+                mbar_arrive(&sm.full[s]);
+            }
+        }
+    }
+    return __shfl_sync(0xffffffffu, ok, 0) != 0;
+}
+
+// Producer lane 0: start id chunk k of the scan (ids [k * kIdChunk, ...)), the u-th
+// chunk of the CTA, into id stage u % kIdRing. An odd count leaves its last id to a
+// plain load (bulk sizes are multiples of 16).
+__device__ __forceinline__ void issue_ids(BulkSmem &sm, const int64_t *__restrict__ slots, int64_t n, int64_t k,
+                                          int64_t u) {
+    const int s = static_cast<int>(u % kIdRing);
+    const int64_t c0 = k * kIdChunk;
+    const int64_t cnt = n - c0 < kIdChunk ? n - c0 : kIdChunk;
+    const uint32_t bytes = static_cast<uint32_t>((cnt & ~static_cast<int64_t>(1)) * 8);
+    if (bytes == 0) {
+        mbar_arrive(&sm.idfull[s]);
+    } else {
+        mbar_arrive_expect_tx(&sm.idfull[s], bytes);
+        bulk_g2s(sm.ids[s], slots + c0, bytes, &sm.idfull[s]);
+    }
+}
+
+template <typename TS>
+__global__ void __launch_bounds__(kBulkThreads, 2)
+    smc_consolidate_bulk_kernel(float *__restrict__ sem, int64_t n_slots, int64_t elems,
+                                const TS *__restrict__ states, const int64_t *__restrict__ slots,
+                                int64_t n, float alpha, int64_t ntiles, int64_t per_cta) {
+    constexpr int CH = 16 / static_cast<int>(sizeof(TS));          // state elements per 16-byte chunk
+    constexpr int64_t R = kStageBytes / static_cast<int64_t>(sizeof(TS));  // elements per tile
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    BulkSmem &sm = *reinterpret_cast<BulkSmem *>(smem_raw);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int64_t nranges = (elems + R - 1) / R;
+    const int64_t t_begin = static_cast<int64_t>(blockIdx.x) * per_cta;
+    const int64_t t_end = t_begin + per_cta < ntiles ? t_begin + per_cta : ntiles;
+    if (tid == 0) {
+        for (int s = 0; s < kRing; ++s) {
+            mbar_init(&sm.full[s], 1);
+            mbar_init(&sm.empty[s], kBulkConsumers / 32);
+        }
+        for (int s = 0; s < kIdRing; ++s) mbar_init(&sm.idfull[s], 1);
+        sm.abort = 0;
+        fence_barrier_init();
+    }
+    __syncthreads();
+
+    if (warp == kBulkConsumers / 32) {
+        // ---- producer warp ----
+        uint32_t g = 0;        // ring stages produced
+        int64_t kid = 0;       // id chunks consumed (all tiles)
+        int64_t kid_issued = 0;
+        bool ok = true;
+        const int64_t nchunks = (n + kIdChunk - 1) / kIdChunk;
+        for (int64_t t = t_begin; t < t_end && ok; ++t) {
+            const int64_t slot = t / nranges;
+            const int64_t e0 = (t % nranges) * R;
+            const int64_t rlen = elems - e0 < R ? elems - e0 : R;
+            const uint32_t bytes = static_cast<uint32_t>(rlen * static_cast<int64_t>(sizeof(TS)));
+            const TS *src = states + e0;
+            const bool flagger = t == 0;
+            const int64_t base = kid;
+            const int64_t first = nchunks < kIdRing ? nchunks : kIdRing;
+            if (lane == 0) {
+                fence_proxy_async_smem();   // the previous tile's reads of the id stages precede their refill
+                for (int64_t k = 0; k < first; ++k) issue_ids(sm, slots, n, k, base + k);
+            }
+            kid_issued = base + first;
+            for (int64_t k = 0; k < nchunks && ok; ++k, ++kid) {
+                const int is = static_cast<int>(kid % kIdRing);
+                int waited = 1;
+                if (lane == 0) waited = wait_or_abort(&sm.idfull[is], static_cast<uint32_t>((kid / kIdRing) & 1), &sm.abort);
+                if (__shfl_sync(0xffffffffu, waited, 0) == 0) {
+                    ok = false;
+                    break;
+                }
+                const int64_t c0 = k * kIdChunk;
+                const int64_t cnt = n - c0 < kIdChunk ? n - c0 : kIdChunk;
+                const int64_t cnt_even = cnt & ~static_cast<int64_t>(1);
+#pragma unroll
+                for (int p = 0; p < kIdChunk / 32; ++p) {
+                    const int j = p * 32 + lane;
+                    const int64_t id = j < cnt_even ? sm.ids[is][j] : (j < cnt ? slots[c0 + j] : -1);
+                    if (flagger && (id >= n_slots || id < -1)) atomicOr(&g_smc_status, PRECOG_DEV_BAD_INDEX);
+                    uint32_t ball = __ballot_sync(0xffffffffu, id == slot);
+                    while (ball != 0u && ok) {
+                        const int jj = __ffs(static_cast<int>(ball)) - 1;
+                        ball &= ball - 1u;
+                        ok = produce_stage(sm, g, lane, src + (c0 + p * 32 + jj) * elems, bytes);
+                        if (ok) ++g;
+                    }
+                }
+                __syncwarp();
+                if (ok && k + kIdRing < nchunks) {
+                    if (lane == 0) {
+                        fence_proxy_async_smem();   // the warp's reads of this id stage precede its refill
+                        issue_ids(sm, slots, n, k + kIdRing, base + k + kIdRing);
+                    }
+                    ++kid_issued;
+                }
+            }
+            if (ok) {
+                ok = produce_stage(sm, g, lane, nullptr, 0);
+                if (ok) ++g;
+            }
+        }
+        if (!ok && lane == 0) {
+            // Give up: record it, stop the consumers, let the issued copies land.
+            atomicOr(&g_smc_status, PRECOG_DEV_TIMEOUT);
+            *static_cast<volatile int32_t *>(&sm.abort) = 1;
+            for (uint32_t g2 = g > kRing ? g - kRing : 0; g2 < g; ++g2)
+                mbar_wait(&sm.full[g2 % kRing], (g2 / kRing) & 1u);
+            for (int64_t u = kid; u < kid_issued; ++u)
+                mbar_wait(&sm.idfull[u % kIdRing], static_cast<uint32_t>((u / kIdRing) & 1));
+        }
+        return;
+    }
+
+    // ---- consumer warps ----
+    const float keep = 1.f - alpha;
+    uint32_t g = 0;
+    for (int64_t t = t_begin; t < t_end; ++t) {
+        const int64_t slot = t / nranges;
+        const int64_t e0 = (t % nranges) * R;
+        const int64_t rlen = elems - e0 < R ? elems - e0 : R;
+        float *srow = sem + slot * elems + e0;
+        float v[kChunksPerThread][CH];
+        bool have[kChunksPerThread];
+#pragma unroll
+        for (int i = 0; i < kChunksPerThread; ++i) {
+            const int64_t q = static_cast<int64_t>(i) * kBulkConsumers + tid;
+            have[i] = q * CH < rlen;
+#pragma unroll
+            for (int k = 0; k < CH; k += 4) {
+                float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (have[i]) f = *reinterpret_cast<const float4 *>(srow + q * CH + k);
+                v[i][k] = f.x;
+                v[i][k + 1] = f.y;
+                v[i][k + 2] = f.z;
+                v[i][k + 3] = f.w;
+            }
+        }
+        bool touched = false;
+        while (true) {
+            const int s = static_cast<int>(g % kRing);
+            if (!wait_or_abort(&sm.full[s], (g / kRing) & 1u, &sm.abort)) {
+                if (lane == 0) atomicOr(&g_smc_status, PRECOG_DEV_TIMEOUT);
+                *static_cast<volatile int32_t *>(&sm.abort) = 1;
+                return;
+            }
+            const int32_t tag = sm.tag[s];
+            if (tag == kTagData) {
+#pragma unroll
+                for (int i = 0; i < kChunksPerThread; ++i) {
+                    if (!have[i]) continue;
+                    const uint4 raw = *reinterpret_cast<const uint4 *>(
+                        sm.ring[s] + (static_cast<int>(i) * kBulkConsumers + tid) * 16);
+                    float h[CH];
+                    if constexpr (std::is_same<TS, float>::value) {
+                        h[0] = __uint_as_float(raw.x);
+                        h[1] = __uint_as_float(raw.y);
+                        h[2] = __uint_as_float(raw.z);
+                        h[3] = __uint_as_float(raw.w);
+                    } else {
+                        const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            h[2 * k] = __uint_as_float(w[k] << 16);
+                            h[2 * k + 1] = __uint_as_float(w[k] & 0xffff0000u);
+                        }
+                    }
+#pragma unroll
+                    for (int k = 0; k < CH; ++k) v[i][k] = fmaf(keep, v[i][k], alpha * h[k]);
+                }
+                touched = true;
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sm.empty[s]);
+            ++g;
+            if (tag != kTagData) break;
+        }
+        if (touched) {
+#pragma unroll
+            for (int i = 0; i < kChunksPerThread; ++i) {
+                if (!have[i]) continue;
+                const int64_t q = static_cast<int64_t>(i) * kBulkConsumers + tid;
+#pragma unroll
+                for (int k = 0; k < CH; k += 4)
+                    *reinterpret_cast<float4 *>(srow + q * CH + k) =
+                        make_float4(v[i][k], v[i][k + 1], v[i][k + 2], v[i][k + 3]);
+            }
+        }
+    }
+}
+
 }  // namespace
 
 cudaError_t launch_smc_route(const void *emb, int dtype, int64_t n, int dim, const void *dom, int M,
@@ -369,8 +622,36 @@ cudaError_t launch_smc_consolidate(float *sem, int64_t n_slots, int64_t elems, c
     const int64_t blocks = (elems / vec + kConsThreads - 1) / kConsThreads;
     if (blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
     const unsigned grid = static_cast<unsigned>(blocks);
-    // Few slots: one CTA per (slot, element range). Each CTA reads all n slot ids (from
+    // Few slots: CTAs per (slot, element range). Each tile reads all n slot ids (from
     // L2), n_slots / 512 of the state bytes for bf16 states, so it pays up to 256 slots.
+    // Whole 16-byte chunks per state row: the states stream through the TMA ring.
+    const int64_t chunk = states_dtype == PRECOG_BF16 ? 8 : 4;
+    if (n_slots >= 1 && n_slots <= 256 && elems % chunk == 0 && reinterpret_cast<uintptr_t>(slots) % 16 == 0) {
+        const int64_t range = kStageBytes / (states_dtype == PRECOG_BF16 ? 2 : 4);
+        const int64_t ntiles = n_slots * ((elems + range - 1) / range);
+        const int64_t resident = 2 * static_cast<int64_t>(device_sm_count());
+        const int64_t per_cta = (ntiles + resident - 1) / resident;
+        const int64_t blocks2 = (ntiles + per_cta - 1) / per_cta;
+        if (blocks2 > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+        const int smem = static_cast<int>(sizeof(BulkSmem));
+        cudaError_t e;
+        if (states_dtype == PRECOG_BF16) {
+            static int attr_bf16 = 0;
+            e = ensure_smem(reinterpret_cast<const void *>(smc_consolidate_bulk_kernel<__nv_bfloat16>), &attr_bf16, smem);
+            if (e != cudaSuccess) return e;
+            smc_consolidate_bulk_kernel<__nv_bfloat16><<<static_cast<unsigned>(blocks2), kBulkThreads, smem, stream>>>(
+                sem, n_slots, elems, static_cast<const __nv_bfloat16 *>(states), slots, n, alpha, ntiles, per_cta);
+        } else {
+            static int attr_f32 = 0;
+            e = ensure_smem(reinterpret_cast<const void *>(smc_consolidate_bulk_kernel<float>), &attr_f32, smem);
+            if (e != cudaSuccess) return e;
+            smc_consolidate_bulk_kernel<float><<<static_cast<unsigned>(blocks2), kBulkThreads, smem, stream>>>(
+                sem, n_slots, elems, static_cast<const float *>(states), slots, n, alpha, ntiles, per_cta);
+        }
+        e = cudaGetLastError();
+        if (e == cudaSuccess) count_launches(1);
+        return e;
+    }
     if (n_slots >= 1 && n_slots <= 256) {
         const int64_t per_cta = static_cast<int64_t>(kSlotThreads) * kSlotItems * vec;
         const dim3 g2(static_cast<unsigned>((elems + per_cta - 1) / per_cta), static_cast<unsigned>(n_slots));

@@ -104,24 +104,60 @@ def test_consolidate_deposit_patterns(cuda_device, n, n_slots, pattern):
         assert rel_err(got[s], ref[s]) < TOL_F32, s
 
 
-def test_consolidate_flags_slot_outside_table(cuda_device):
-    """A slot >= n_slots deposits nothing and raises PRECOG_DEV_BAD_INDEX; the other
-    deposits still apply."""
+@pytest.mark.parametrize("elems,n_slots", [(64, 3), (63, 3), (64, 300)])
+def test_consolidate_flags_slot_outside_table(cuda_device, elems, n_slots):
+    """A slot >= n_slots or below -1 deposits nothing and raises PRECOG_DEV_BAD_INDEX;
+    the other deposits still apply (the staged per-slot fold, the register per-slot fold
+    for a row of odd length, the batch fold for a table of more than 256 slots)."""
     import torch
     import paper_2608_02560_gb300 as pg
     rng = np.random.default_rng(5)
-    states = rng.standard_normal((6, 64)).astype(np.float32)
-    slot_np = np.array([0, 1, 9, 1, 0, 2], dtype=np.int64)      # 9 is outside a 3-slot table
-    sem0 = np.zeros((3, 64), dtype=np.float32)
+    states = rng.standard_normal((7, elems)).astype(np.float32)
+    slot_np = np.array([0, 1, n_slots + 6, 1, 0, -2, 2], dtype=np.int64)
+    sem0 = np.zeros((n_slots, elems), dtype=np.float32)
     sem = torch.from_numpy(sem0).to(cuda_device)
     pg.precog_smc_consolidate(sem, torch.from_numpy(states).to(cuda_device),
                               torch.from_numpy(slot_np).to(cuda_device), 0.5)
     st, bits = pg.precog_device_status()
     assert st != 0 and bits & pg.PRECOG_DEV_BAD_INDEX
     keep = slot_np.copy()
-    keep[2] = -1
+    keep[2] = keep[5] = -1
     ref = oracle.smc_consolidate(sem0, states, keep, 0.5)
     assert rel_err(to_np(sem), ref) < TOL_F32
+
+
+@pytest.mark.parametrize("dtype,elems,n,n_slots,pattern", [
+    ("f32", 4132, 200, 64, "cyclic"), ("bf16", 4200, 77, 3, "runs"), ("bf16", 8, 1, 5, "cyclic"),
+    ("f32", 4, 96, 40, "random"), ("bf16", 4200, 2500, 7, "random"), ("bf16", 12296, 600, 256, "random"),
+    ("f32", 2048, 300, 1, "runs"), ("f32", 6148, 1030, 100, "random")])
+def test_consolidate_staged_patterns(cuda_device, dtype, elems, n, n_slots, pattern):
+    """The fold that streams states through the shared-memory ring (rows of whole
+    16-byte chunks, at most 256 slots): element ranges of 2048 (fp32) or 4096 (bf16)
+    with a ragged last range, several tiles per CTA (256 slots x 4 ranges), more slot
+    ids than one prefetch window (512), one slot, a single deposit, -1 mixed in."""
+    import torch
+    import paper_2608_02560_gb300 as pg
+    rng = np.random.default_rng(elems + n + n_slots)
+    states = rng.standard_normal((n, elems)).astype(np.float32)
+    if dtype == "bf16":
+        states_dev = torch.from_numpy(states).to(cuda_device).to(torch.bfloat16)
+        states = states_dev.float().cpu().numpy()
+    else:
+        states_dev = torch.from_numpy(states).to(cuda_device)
+    if pattern == "cyclic":
+        slot_np = np.arange(n, dtype=np.int64) % n_slots
+    elif pattern == "runs":
+        slot_np = (np.arange(n, dtype=np.int64) // 10) % n_slots
+    else:
+        slot_np = rng.integers(-1, n_slots, size=n).astype(np.int64)
+    sem0 = rng.standard_normal((n_slots, elems)).astype(np.float32)
+    sem = torch.from_numpy(sem0).to(cuda_device)
+    pg.precog_smc_consolidate(sem, states_dev, torch.from_numpy(slot_np).to(cuda_device), 0.3)
+    assert pg.precog_device_status()[0] == 0
+    ref = oracle.smc_consolidate(sem0, states, slot_np, 0.3)
+    got = to_np(sem)
+    for s in range(n_slots):
+        assert rel_err(got[s], ref[s]) < TOL_F32, s
 
 
 def test_smc_benchmark_sizes_sampled(cuda_device):
