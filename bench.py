@@ -88,6 +88,29 @@ def peaks():
     return FALLBACK_HBM_GBS, "fallback"
 
 
+# FP32 lane operations one channel-token of the rescaled capture needs on the FMA pipe:
+# the exponent sum L += dt * k (1), u = dt * x (1), the 16 weights u * E^(n+1) (16
+# multiplies) and the 16 accumulations G_n += w_n * B_n (16 FMAs). The exponential E = 2^L
+# runs on the SFU and is not counted.
+ALU_OPS_PER_CHANNEL_TOKEN = 34
+FP32_LANES_PER_SM = 128      # 4 sub-partitions x 32 FP32 lanes (FFMA and FFMA2 alike)
+FALLBACK_SM_MHZ = 2070.0
+
+
+def alu_peak_tops(dev):
+    """FP32 FMA-pipe peak in tera lane-operations per second: SMs x lanes x max SM clock."""
+    import torch
+    mhz = FALLBACK_SM_MHZ
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        try:
+            mhz = float(json.load(open(path)).get("sm_max_mhz", mhz))
+        except Exception:
+            pass
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    return sms * FP32_LANES_PER_SM * mhz * 1e6 / 1e12, sms, mhz
+
+
 def profiled_traffic():
     """DRAM traffic of one single-layer encode launch from the committed ncu summary, if
     it was taken on the current scan kernel source (else None)."""
@@ -577,10 +600,22 @@ def main():
     avg_scan_ms = statistics.mean(scan_ms)
     achieved = bpl / (avg_scan_ms * 1e-3) / 1e9
     layer_traffic = profiled_traffic()
-    roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                "frac": achieved / hbm, "traffic": None if layer_traffic is None else S * layer_traffic,
+    # The scan is bound by the FP32 FMA pipe (ncu: FMA pipe 66 % busy, DRAM 36 %), so the
+    # roofline is the ALU one; the HBM fraction the metric names is carried beside it.
+    alu_peak, sms, mhz = alu_peak_tops(dev)
+    ops = S * T * D * ALU_OPS_PER_CHANNEL_TOKEN
+    alu_achieved = ops / (avg_scan_ms * 1e-3) / 1e12
+    roofline = {"bound": "alu", "achieved": alu_achieved, "peak": alu_peak,
+                "unit": "Tops/s (FP32 FMA-pipe lane operations)", "frac": alu_achieved / alu_peak,
+                "traffic": None if layer_traffic is None else S * layer_traffic,
+                "peak_derivation": f"{sms} SMs x {FP32_LANES_PER_SM} FP32 lanes x {mhz:.0f} MHz",
+                "ops_per_channel_token": ALU_OPS_PER_CHANNEL_TOKEN, "algorithmic_ops_per_launch": ops,
+                "hbm": {"achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+                        "peak_source": peak_src,
+                        "alu_ceiling_frac": alu_peak * 1e12 / ALU_OPS_PER_CHANNEL_TOKEN
+                        * (bpl / (S * T * D)) / (hbm * 1e9)},
                 "layers_per_launch": S,
-                "kernel": "scan_kernel (encode, capture)", "peak_source": peak_src,
+                "kernel": "scan_kernel (encode, capture)",
                 "algorithmic_bytes_per_launch": bpl, "avg_launch_ms": avg_scan_ms}
 
     # ---------------- end to end: host inputs -> device -> encode/query -> host results

@@ -60,7 +60,8 @@ __device__ uint32_t g_scan_status;
 #endif
 
 constexpr int kN = 16;          // state size (N) supported by the kernels
-constexpr int kMaxSlice = 256;  // channels per CTA at most
+constexpr int kMaxSlice = 256;  // channels per CTA at most (the default slice)
+constexpr int kWideSlice = 512; // rows of up to this many channels are staged whole
 constexpr int kBarBytes = 128;  // barrier area at the start of shared memory
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr int kMaxTopk = 8;     // states composed at most by one injection
@@ -73,13 +74,21 @@ enum Mode { kGeneral = 0, kPower = 1 };
 constexpr int kTrajNone = 0, kTrajDirect = 1, kTrajRescaled = 2;
 
 template <typename TIn_, bool HAS_Y_, bool HAS_H0_, int MODE_, int CPT_, int TILE_, int STAGES_,
-          int MINB_, int TRAJ_ = kTrajNone>
+          int MINB_, int TRAJ_ = kTrajNone, int MAXSLICE_ = kMaxSlice>
 struct Cfg {
     using TIn = TIn_;
+    // Widest channel slice of one CTA. Each CTA stages its slice of every token row; a
+    // slice narrower than the row turns the row into separate pieces, and HBM serves
+    // short scattered pieces far below its streaming rate, so rows up to 512 channels
+    // stay whole. MINB counts resident CTAs of kMaxSlice channels (the register budget
+    // per thread), whatever the slice.
+    static constexpr int MAXSLICE = MAXSLICE_;
+    static constexpr int LB_THREADS = MAXSLICE_ / CPT_;
+    static constexpr int LB_BLOCKS = MINB_ * kMaxSlice / MAXSLICE_ > 0 ? MINB_ * kMaxSlice / MAXSLICE_ : 1;
     static constexpr bool HAS_Y = HAS_Y_, HAS_H0 = HAS_H0_;
     // keep every stride-th state (K-dial, Sec. 5.2), with the direct or the rescaled update
     static constexpr int TRAJ = TRAJ_;
-    static constexpr int MODE = MODE_, CPT = CPT_, TILE = TILE_, STAGES = STAGES_, MINB = MINB_;
+    static constexpr int MODE = MODE_, CPT = CPT_, TILE = TILE_, STAGES = STAGES_;
     static constexpr bool CONV = !std::is_same<TIn_, float>::value;
     static constexpr int SZ = sizeof(TIn_);
     static constexpr bool RESCALED = MODE_ == kPower && !HAS_Y_ && TRAJ_ != kTrajDirect;
@@ -460,7 +469,7 @@ __device__ __forceinline__ void scan_tile_rescaled(const unsigned char *st, cons
 
 // ---------------------------------------------------------------------------
 template <class C>
-__global__ void __launch_bounds__(kMaxSlice / C::CPT, C::MINB)
+__global__ void __launch_bounds__(C::LB_THREADS, C::LB_BLOCKS)
     scan_kernel(const ScanParams p, const int DS, const int slices) {
     using TIn = typename C::TIn;
     constexpr int CPT = C::CPT, TILE = C::TILE, STAGES = C::STAGES, SZ = C::SZ;
@@ -731,12 +740,12 @@ __global__ void __launch_bounds__(kMaxSlice / C::CPT, C::MINB)
     }
 }
 
-// Widest channel slice (<= kMaxSlice channels, 16-byte rows) that divides D
+// Widest channel slice (<= maxslice channels, 16-byte rows) that divides D
 // into whole threads of CPT channels.
-int pick_slice(int D, int sz, int cpt) {
-    const int cands[] = {256, 128, 64, 32, 16, 8, 4, 2};
+int pick_slice(int D, int sz, int cpt, int maxslice) {
+    const int cands[] = {512, 256, 128, 64, 32, 16, 8, 4, 2};
     for (int ds : cands)
-        if (ds <= kMaxSlice && D % ds == 0 && (ds * sz) % 16 == 0 && ds % cpt == 0) return ds;
+        if (ds <= maxslice && D % ds == 0 && (ds * sz) % 16 == 0 && ds % cpt == 0) return ds;
     return 0;
 }
 
@@ -749,7 +758,7 @@ bool few_items(const ScanParams &p) {
 
 template <class C>
 cudaError_t launch_cfg(const ScanParams &p, cudaStream_t stream) {
-    const int DS = pick_slice(p.D, C::SZ, C::CPT);
+    const int DS = pick_slice(p.D, C::SZ, C::CPT, C::MAXSLICE);
     if (DS == 0) return cudaErrorInvalidValue;
     const int slices = p.D / DS;
     const StageLayout lay = stage_layout(C::TILE, DS, C::SZ, C::HAS_Y, C::CONV);
@@ -773,17 +782,17 @@ template <typename TIn, bool HAS_Y, bool HAS_H0, int MODE, int TRAJ = kTrajNone>
 cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
     if constexpr (TRAJ == kTrajRescaled) {
         return launch_cfg<Cfg<TIn, false, false, kPower, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
-                              PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB, kTrajRescaled>>(p, stream);
+                              PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB, kTrajRescaled, kWideSlice>>(p, stream);
     } else if constexpr (TRAJ == kTrajDirect) {
         // short strides and general A: the direct update (h is at hand after every token)
         if constexpr (MODE == kPower)
             return launch_cfg<Cfg<TIn, false, false, MODE, PRECOG_DIRECT_CPT, PRECOG_DIRECT_TILE,
-                                  PRECOG_DIRECT_STAGES, PRECOG_DIRECT_MINB, kTrajDirect>>(p, stream);
+                                  PRECOG_DIRECT_STAGES, PRECOG_DIRECT_MINB, kTrajDirect, kWideSlice>>(p, stream);
         else
             return launch_cfg<Cfg<TIn, false, false, MODE, 2, 16, 4, 3, kTrajDirect>>(p, stream);
     } else if constexpr (MODE == kPower && !HAS_Y) {
         return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
-                              PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB>>(p, stream);
+                              PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB, kTrajNone, kWideSlice>>(p, stream);
     } else {
         if constexpr (MODE == kPower) {
             // Fewer work items than SMs (a single query's prefill: one CTA per layer) is a
@@ -792,7 +801,7 @@ cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
             if (few_items(p))
                 return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, 2, 16, 2, 3>>(p, stream);
             return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, PRECOG_DIRECT_CPT, PRECOG_DIRECT_TILE,
-                                  PRECOG_DIRECT_STAGES, PRECOG_DIRECT_MINB>>(p, stream);
+                                  PRECOG_DIRECT_STAGES, PRECOG_DIRECT_MINB, kTrajNone, kWideSlice>>(p, stream);
         } else {
             // general A keeps 16 exponent coefficients per channel: 2 channels per thread
             return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, 2, 16, 4, 3>>(p, stream);

@@ -139,11 +139,12 @@ def test_multi_layer_call_and_layer_offset(cuda_device):
             assert rel_err(got[c, 2 + l], ref[c]) < TOL_F32
 
 
-@pytest.mark.parametrize("D,y_mode", [(512, False), (512, True), (768, True)])
+@pytest.mark.parametrize("D,y_mode", [(512, False), (1024, False), (1024, True), (768, True)])
 def test_multi_layer_sliced_channels(cuda_device, D, y_mode):
-    """Channels wider than one CTA's 256-channel slice, three layers in one call: each CTA
-    stages its slice of x and dt through a 3-D tensor map (channel, row, layer); chunks
-    end inside and at the end of 16-row tiles. Every layer's states (and y) vs the oracle."""
+    """Rows wider than one CTA's channel slice (512 channels with the power-form A, 256
+    where 512 does not divide D), three layers in one call: each CTA stages its slice of
+    every x and dt row with one bulk copy per row; D = 512 stays one slice. Chunks end
+    inside and at the end of 16-row tiles. Every layer's states (and y) vs the oracle."""
     import torch
     pg = _pg()
     d = cuda_device
@@ -225,14 +226,15 @@ def test_deterministic(cuda_device):
 
 def test_power_statement_is_verified(cuda_device):
     """a_kind = PRECOG_A_POWER with an A that is not (n+1)*A[d,0]: nothing is written for
-    the affected channel blocks and PRECOG_DEV_BAD_A is flagged; A[d,0] > 0 as well."""
+    the affected channel blocks and PRECOG_DEV_BAD_A is flagged; A[d,0] > 0 as well. A
+    1024-channel layer is encoded in two blocks of 512 channels."""
     import torch
     pg = _pg()
     d = cuda_device
-    T, D, N = 50, 512, 16
+    T, D, N = 50, 1024, 16
     x, dt, A, B, _ = synth.host_scan_inputs(T, D, N, seed=2)
     A_bad = A.copy()
-    A_bad[300, 5] *= 1.5                    # channel 300 sits in the second 256-channel block
+    A_bad[600, 5] *= 1.5                    # channel 600 sits in the second 512-channel block
     off = _t(np.array([0, T], dtype=np.int64), d, torch.int64)
     for Ab in (A_bad, -A):
         states = torch.full((1, 1, D, N), 3.0, dtype=torch.float32, device=d)
@@ -240,13 +242,13 @@ def test_power_statement_is_verified(cuda_device):
                                                a_kind=pg.PRECOG_A_POWER), off, T, states_out=states)
         st, bits = pg.precog_device_status()
         assert st == 5 and bits == pg.PRECOG_DEV_BAD_A
-        assert torch.all(states[0, 0, 256:] == 3.0)
+        assert torch.all(states[0, 0, 512:] == 3.0)
     ref, _ = oracle.rollout(x, dt, A, B)
     states = torch.full((1, 1, D, N), 3.0, dtype=torch.float32, device=d)
     pg.precog_encode_chunks(pg.scan_inputs(_t(x, d), _t(dt, d), _t(B, d), _t(A_bad, d),
                                            a_kind=pg.PRECOG_A_POWER), off, T, states_out=states)
     pg.precog_device_status()
-    assert rel_err(to_np(states[0, 0, :256]), ref[:256]) < TOL_F32   # the valid block is done
+    assert rel_err(to_np(states[0, 0, :512]), ref[:512]) < TOL_F32   # the valid block is done
 
 
 @pytest.mark.parametrize("scale,dt_shift", [(1.0, -2.0), (40.0, -2.0), (1.0, 2.5), (0.02, -4.0)])
