@@ -456,7 +456,9 @@ def measure_extensions(pg, synth, torch, dev, layer_in, off, T, n_chunks, index,
     os_ = torch.empty(n_emb, dtype=torch.int64, device=dev)
     ms = timed(lambda: pg.precog_smc_route(emb, dom, sub, Jt, om, oj, os_))
     out["smc_route_4096x(16+64)"] = dict(ms=ms, flops=2.0 * n_emb * (Md + J) * dim,
-                                         note="latency-bound: 80 dependent 768-dim dots per warp")
+                                         l2_to_sm_bytes=n_emb * (Md + J) * dim * 2,
+                                         note="each warp streams its embedding's 80 prototypes "
+                                              "(120 KB) from L2, eight at a time")
     bank_states = qbank[:n_emb].view(n_emb, -1)
     sem = torch.zeros((J, bank_states.shape[1]), dtype=torch.float32, device=dev)
     slots = torch.arange(n_emb, dtype=torch.int64, device=dev) % J

@@ -17,22 +17,57 @@ __device__ uint32_t g_smc_status;
 
 constexpr int kRouteWarps = 8;
 
-template <typename T>
-__device__ __forceinline__ float dot_warp(const T *__restrict__ a, const T *__restrict__ b, int dim,
-                                          int lane) {
-    // fixed lane mapping and butterfly: the same two vectors always give the same score
-    float acc = 0.f;
-    for (int k = lane; k < dim; k += 32) acc = fmaf(to_f32(a[k]), to_f32(b[k]), acc);
+constexpr int kRouteP = 8;   // prototypes scored per pass
+
+// acc[p] = <e, protos[p]> for p < count (<= kRouteP prototypes, `stride` elements
+// apart). Each lane sums a fixed subset of the coordinates in a fixed order -- 16-byte
+// vectors v = lane, lane + 32, ... when VEC, single elements otherwise -- and a fixed
+// xor butterfly adds the lanes, so the same two vectors always give the same score
+// and every lane holds it. The count prototypes' loads of a vector are in flight
+// together.
+template <typename T, bool VEC>
+__device__ __forceinline__ void dots_warp(const T *__restrict__ e, const T *__restrict__ protos, int64_t stride,
+                                          int count, int dim, int lane, float (&acc)[kRouteP]) {
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    return acc;
+    for (int q = 0; q < kRouteP; ++q) acc[q] = 0.f;
+    if constexpr (VEC) {
+        constexpr int EL = 16 / static_cast<int>(sizeof(T));
+        const int nvec = dim / EL;
+        for (int v = lane; v < nvec; v += 32) {
+            const uint4 ev = *reinterpret_cast<const uint4 *>(e + static_cast<int64_t>(v) * EL);
+            uint4 pv[kRouteP];
+#pragma unroll
+            for (int q = 0; q < kRouteP; ++q)
+                if (q < count) pv[q] = *reinterpret_cast<const uint4 *>(protos + q * stride + static_cast<int64_t>(v) * EL);
+            const T *ee = reinterpret_cast<const T *>(&ev);
+#pragma unroll
+            for (int q = 0; q < kRouteP; ++q) {
+                if (q >= count) break;
+                const T *pp = reinterpret_cast<const T *>(&pv[q]);
+#pragma unroll
+                for (int k = 0; k < EL; ++k) acc[q] = fmaf(to_f32(ee[k]), to_f32(pp[k]), acc[q]);
+            }
+        }
+    } else {
+        for (int k = lane; k < dim; k += 32) {
+            const float ek = to_f32(e[k]);
+#pragma unroll
+            for (int q = 0; q < kRouteP; ++q)
+                if (q < count) acc[q] = fmaf(ek, to_f32(protos[q * stride + k]), acc[q]);
+        }
+    }
+#pragma unroll
+    for (int q = 0; q < kRouteP; ++q)
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) acc[q] += __shfl_xor_sync(0xffffffffu, acc[q], o);
 }
 
 // One warp per embedding: the best domain prototype, then the best of that
-// domain's J[m] sub-cluster prototypes (strict '>': lowest index on ties, NaN
-// never wins). slot = m * J_max + j, or -1 when no comparable score exists.
-template <typename T>
-__global__ void __launch_bounds__(kRouteWarps * 32)
+// domain's J[m] sub-cluster prototypes (strict '>' in index order: lowest index on
+// ties, NaN never wins). slot = m * J_max + j, or -1 when no comparable score exists.
+// VEC: rows are whole 16-byte vectors on 16-byte boundaries.
+template <typename T, bool VEC>
+__global__ void __launch_bounds__(kRouteWarps * 32, 3)
     smc_route_kernel(const T *__restrict__ emb, int64_t n, int dim, const T *__restrict__ dom, int M,
                      const T *__restrict__ sub, int J_max, const int32_t *__restrict__ J,
                      int32_t *__restrict__ out_m, int32_t *__restrict__ out_j,
@@ -41,14 +76,18 @@ __global__ void __launch_bounds__(kRouteWarps * 32)
     const int64_t c = static_cast<int64_t>(blockIdx.x) * kRouteWarps + (threadIdx.x >> 5);
     if (c >= n) return;
     const T *e = emb + c * dim;
+    float acc[kRouteP];
     float best = -__int_as_float(0x7f800000);
     int m = -1;
-    for (int i = 0; i < M; ++i) {
-        const float s = dot_warp(e, dom + static_cast<int64_t>(i) * dim, dim, lane);
-        if (s > best) {
-            best = s;
-            m = i;
-        }
+    for (int i0 = 0; i0 < M; i0 += kRouteP) {
+        const int cnt = M - i0 < kRouteP ? M - i0 : kRouteP;
+        dots_warp<T, VEC>(e, dom + static_cast<int64_t>(i0) * dim, dim, cnt, dim, lane, acc);
+#pragma unroll
+        for (int q = 0; q < kRouteP; ++q)
+            if (q < cnt && acc[q] > best) {
+                best = acc[q];
+                m = i0 + q;
+            }
     }
     int j = -1;
     if (m >= 0) {
@@ -58,12 +97,16 @@ __global__ void __launch_bounds__(kRouteWarps * 32)
             Jm = 0;
         }
         best = -__int_as_float(0x7f800000);
-        for (int i = 0; i < Jm; ++i) {
-            const float s = dot_warp(e, sub + (static_cast<int64_t>(m) * J_max + i) * dim, dim, lane);
-            if (s > best) {
-                best = s;
-                j = i;
-            }
+        const T *sm_ = sub + static_cast<int64_t>(m) * J_max * dim;
+        for (int i0 = 0; i0 < Jm; i0 += kRouteP) {
+            const int cnt = Jm - i0 < kRouteP ? Jm - i0 : kRouteP;
+            dots_warp<T, VEC>(e, sm_ + static_cast<int64_t>(i0) * dim, dim, cnt, dim, lane, acc);
+#pragma unroll
+            for (int q = 0; q < kRouteP; ++q)
+                if (q < cnt && acc[q] > best) {
+                    best = acc[q];
+                    j = i0 + q;
+                }
         }
     }
     if (lane == 0) {
@@ -586,6 +629,24 @@ __global__ void __launch_bounds__(kBulkThreads, 2)
 
 }  // namespace
 
+template <typename T>
+void launch_route_t(const void *emb, int64_t n, int dim, const void *dom, int M, const void *sub, int J_max,
+                    const int32_t *J, int32_t *out_m, int32_t *out_j, int64_t *out_slot, unsigned grid,
+                    cudaStream_t stream) {
+    const auto *e = static_cast<const T *>(emb);
+    const auto *d = static_cast<const T *>(dom);
+    const auto *s = static_cast<const T *>(sub);
+    const auto a16 = [](const void *ptr) { return reinterpret_cast<uintptr_t>(ptr) % 16 == 0; };
+    const bool vec = (static_cast<int64_t>(dim) * static_cast<int64_t>(sizeof(T))) % 16 == 0 && a16(emb) &&
+                     a16(dom) && a16(sub);
+    if (vec)
+        smc_route_kernel<T, true><<<grid, kRouteWarps * 32, 0, stream>>>(e, n, dim, d, M, s, J_max, J, out_m,
+                                                                        out_j, out_slot);
+    else
+        smc_route_kernel<T, false><<<grid, kRouteWarps * 32, 0, stream>>>(e, n, dim, d, M, s, J_max, J, out_m,
+                                                                         out_j, out_slot);
+}
+
 cudaError_t launch_smc_route(const void *emb, int dtype, int64_t n, int dim, const void *dom, int M,
                              const void *sub, int J_max, const int32_t *J, int32_t *out_m,
                              int32_t *out_j, int64_t *out_slot, cudaStream_t stream) {
@@ -593,19 +654,13 @@ cudaError_t launch_smc_route(const void *emb, int dtype, int64_t n, int dim, con
     const unsigned grid = static_cast<unsigned>((n + kRouteWarps - 1) / kRouteWarps);
     switch (dtype) {
         case PRECOG_F16:
-            smc_route_kernel<__half><<<grid, kRouteWarps * 32, 0, stream>>>(
-                static_cast<const __half *>(emb), n, dim, static_cast<const __half *>(dom), M,
-                static_cast<const __half *>(sub), J_max, J, out_m, out_j, out_slot);
+            launch_route_t<__half>(emb, n, dim, dom, M, sub, J_max, J, out_m, out_j, out_slot, grid, stream);
             break;
         case PRECOG_BF16:
-            smc_route_kernel<__nv_bfloat16><<<grid, kRouteWarps * 32, 0, stream>>>(
-                static_cast<const __nv_bfloat16 *>(emb), n, dim, static_cast<const __nv_bfloat16 *>(dom), M,
-                static_cast<const __nv_bfloat16 *>(sub), J_max, J, out_m, out_j, out_slot);
+            launch_route_t<__nv_bfloat16>(emb, n, dim, dom, M, sub, J_max, J, out_m, out_j, out_slot, grid, stream);
             break;
         default:
-            smc_route_kernel<float><<<grid, kRouteWarps * 32, 0, stream>>>(
-                static_cast<const float *>(emb), n, dim, static_cast<const float *>(dom), M,
-                static_cast<const float *>(sub), J_max, J, out_m, out_j, out_slot);
+            launch_route_t<float>(emb, n, dim, dom, M, sub, J_max, J, out_m, out_j, out_slot, grid, stream);
     }
     cudaError_t e = cudaGetLastError();
     if (e == cudaSuccess) count_launches(1);

@@ -36,6 +36,37 @@ def test_route_exact_integer_scores(cuda_device, dtype_name):
     np.testing.assert_array_equal(slot.cpu().numpy(), exp_slot)
 
 
+@pytest.mark.parametrize("dtype_name,dim", [("float16", 100), ("float32", 61), ("bfloat16", 96)])
+def test_route_nan_prototypes_and_unaligned_rows(cuda_device, dtype_name, dim):
+    """Rows that are not whole 16-byte vectors (element loads) and rows that are, more
+    prototypes than one pass of eight at both levels, and NaN prototypes (a NaN score never
+    wins; an embedding whose domain scores are all NaN routes nowhere)."""
+    import torch
+    import paper_2608_02560_gb300 as pg
+    dtype = getattr(torch, dtype_name)
+    rng = np.random.default_rng(dim)
+    n, M, J_max = 700, 11, 13
+    emb = rng.integers(-2, 3, size=(n, dim)).astype(np.float32)
+    P = rng.integers(-2, 3, size=(M, dim)).astype(np.float32)
+    S = rng.integers(-2, 3, size=(M, J_max, dim)).astype(np.float32)
+    P[4, 7] = np.nan                      # domain 4 never wins
+    S[:, 9, 3] = np.nan                   # sub-cluster 9 of every domain never wins
+    emb[5, :] = np.nan                    # all scores NaN: routes nowhere
+    J = rng.integers(0, J_max + 1, size=M).astype(np.int32)
+    J[0] = J_max
+    t = lambda a, dt=dtype: torch.from_numpy(np.ascontiguousarray(a)).to(cuda_device, dt)
+    dm = torch.empty(n, dtype=torch.int32, device=cuda_device)
+    dj = torch.empty(n, dtype=torch.int32, device=cuda_device)
+    slot = torch.empty(n, dtype=torch.int64, device=cuda_device)
+    pg.precog_smc_route(t(emb), t(P), t(S), t(J, torch.int32), dm, dj, slot)
+    assert pg.precog_device_status()[0] == 0
+    rm, rj = oracle.smc_route(emb, P, S, J)
+    assert rm[5] == -1 and 4 not in set(rm.tolist()) and 9 not in set(rj.tolist())
+    np.testing.assert_array_equal(dm.cpu().numpy(), rm)
+    np.testing.assert_array_equal(dj.cpu().numpy(), rj)
+    np.testing.assert_array_equal(slot.cpu().numpy(), np.where(rj >= 0, rm * J_max + rj, -1))
+
+
 def test_consolidate_then_session_init(cuda_device):
     """Deposit 300 chunk states (bf16, 24 layers of D=256, N=16) into 20 semantic slots
     in order (some forgetting candidates, slot -1), compare the fp32 table with the
