@@ -454,7 +454,10 @@ precog_status precog_device_status(void *stream, uint32_t *bits_out) {
     uint32_t w = 0;
     e = precog::selftest_status_word_read_clear(&w);
     if (e != cudaSuccess) return cuda_fail(e, "read self-test status");
-    *bits_out = a | b | c | z | w;
+    uint32_t l = 0;
+    e = precog::scan_latency_status_word_read_clear(&l);
+    if (e != cudaSuccess) return cuda_fail(e, "read latency scan status");
+    *bits_out = a | b | c | z | w | l;
     if (*bits_out == 0) return ok();
     if (*bits_out & PRECOG_DEV_TIMEOUT)
         return fail(PRECOG_ERR_TIMEOUT, "a device-side wait gave up (bits 0x%x)", *bits_out);

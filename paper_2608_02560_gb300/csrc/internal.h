@@ -69,6 +69,12 @@ void count_launches(uint64_t n);
 cudaError_t ensure_smem(const void *kernel, int *cached_bytes, int bytes);
 
 cudaError_t launch_scan(const ScanParams &p, cudaStream_t stream);
+
+// Latency-shaped direct scan with readout (scan_latency.cu): power-form A, D a
+// multiple of 64; scan.cu routes launches with fewer work items than SMs to it.
+bool scan_latency_eligible(const ScanParams &p);
+cudaError_t launch_scan_latency(const ScanParams &p, cudaStream_t stream);
+cudaError_t scan_latency_status_word_read_clear(uint32_t *bits);
 cudaError_t scan_status_word_read_clear(uint32_t *bits);
 
 struct RetrieveParams {

@@ -796,10 +796,12 @@ cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
     } else {
         if constexpr (MODE == kPower) {
             // Fewer work items than SMs (a single query's prefill: one CTA per layer) is a
-            // latency-bound launch: two channels per thread halve each thread's serial work
-            // per token (measured 27 -> 21 us for 24 layers x 64 tokens).
-            if (few_items(p))
+            // latency-bound launch: the latency-shaped kernel splits every channel's states
+            // over four threads; shapes it does not take run two channels per thread.
+            if (few_items(p)) {
+                if (scan_latency_eligible(p)) return launch_scan_latency(p, stream);
                 return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, 2, 16, 2, 3>>(p, stream);
+            }
             return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, PRECOG_DIRECT_CPT, PRECOG_DIRECT_TILE,
                                   PRECOG_DIRECT_STAGES, PRECOG_DIRECT_MINB, kTrajNone, kWideSlice>>(p, stream);
         } else {

@@ -152,3 +152,70 @@ def test_query_workload_prefill(cuda_device, Q):
                                           to_np(C[l, sl]), h0=h0, want_y=True)
             assert rel_err_stored(to_np(h[q, l]), ref_h) < TOL_BF16
             assert rel_err_stored(to_np(y[l, sl]), ref_y) < TOL_BF16
+
+
+@pytest.mark.parametrize("D,Tq,in32,bank32,y32,st32", [
+    (64, 1, True, True, True, True), (128, 63, False, False, False, False),
+    (512, 65, False, True, True, False), (256, 200, True, False, False, True),
+    (192, 64, False, False, True, True)])
+def test_small_batch_prefill_shapes(cuda_device, D, Tq, in32, bank32, y32, st32):
+    """Prefill launches with fewer (query, layer) items than SMs take the latency-shaped
+    kernel (four threads per channel, 64-channel blocks): one to eight channel blocks,
+    token counts inside one 64-token tile, at its edge and across tiles, fp32 and bf16
+    inputs, banks, readouts and states, an injected row and the zero state (row -1)."""
+    import torch
+    pg = _pg()
+    d = cuda_device
+    N, Q, L = 16, 3, 2
+    f32, b16 = torch.float32, torch.bfloat16
+    idt = f32 if in32 else b16
+    ins = [synth.host_scan_inputs(Q * Tq, D, N, seed=D + Tq + l) for l in range(L)]
+    cast = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(d, idt)
+    st = lambda k: torch.stack([cast(i[k]) for i in ins]).contiguous()
+    x, dt, B, C = st(0), st(1), st(3), st(4)
+    A = torch.from_numpy(np.stack([synth.structured_A(D, N) * (1 + 0.5 * l) for l in range(L)])).to(d)
+    bank = torch.randn((5, L, D, N), device=d).to(f32 if bank32 else b16)
+    idx = torch.tensor([3, -1, 0], dtype=torch.int64, device=d)
+    y = torch.empty((L, Q * Tq, D), dtype=f32 if y32 else b16, device=d)
+    h = torch.empty((Q, L, D, N), dtype=f32 if st32 else b16, device=d)
+    pg.precog_prefill_from_state(pg.scan_inputs(x, dt, B, A, C, a_kind=pg.PRECOG_A_POWER), Q, Tq,
+                                 bank, idx=idx, y_out=y, state_out=h)
+    assert pg.precog_device_status()[0] == 0
+    tol = TOL_F32 if in32 else TOL_BF16
+    cmp_h = rel_err if st32 else rel_err_stored
+    cmp_y = rel_err if y32 else rel_err_stored
+    for q, row in enumerate((3, -1, 0)):
+        for l in range(L):
+            sl = slice(q * Tq, (q + 1) * Tq)
+            h0 = None if row < 0 else to_np(bank[row, l].float())
+            ref_h, ref_y = oracle.rollout(to_np(x[l, sl].float()), to_np(dt[l, sl].float()),
+                                          to_np(A[l]), to_np(B[l, sl].float()), to_np(C[l, sl].float()),
+                                          h0=h0, want_y=True)
+            assert cmp_h(to_np(h[q, l].float()), ref_h) < max(tol, TOL_F32), (q, l)
+            assert cmp_y(to_np(y[l, sl].float()), ref_y) < max(tol, TOL_F32), (q, l)
+
+
+def test_small_batch_prefill_rejects_false_power_statement(cuda_device):
+    """The latency-shaped prefill verifies a_kind = PRECOG_A_POWER per 64-channel block: a
+    block whose A is not (n+1)*A[d,0] writes neither y nor the state and flags
+    PRECOG_DEV_BAD_A; the other blocks are computed."""
+    import torch
+    pg = _pg()
+    d = cuda_device
+    D, N, Tq = 128, 16, 40
+    x, dt, A, B, C = synth.host_scan_inputs(Tq, D, N, seed=31)
+    A_bad = A.copy()
+    A_bad[100, 7] *= 1.25                      # channel 100: second 64-channel block
+    bank = torch.randn((2, 1, D, N), device=d)
+    idx = torch.tensor([1], dtype=torch.int64, device=d)
+    y = torch.full((1, Tq, D), 7.0, dtype=torch.float32, device=d)
+    h = torch.full((1, 1, D, N), 7.0, dtype=torch.float32, device=d)
+    pg.precog_prefill_from_state(pg.scan_inputs(_t(x, d), _t(dt, d), _t(B, d), _t(A_bad, d), _t(C, d),
+                                                a_kind=pg.PRECOG_A_POWER),
+                                 1, Tq, bank, idx=idx, y_out=y, state_out=h)
+    st, bits = pg.precog_device_status()
+    assert st == 5 and bits == pg.PRECOG_DEV_BAD_A
+    assert torch.all(y[0, :, 64:] == 7.0) and torch.all(h[0, 0, 64:] == 7.0)
+    ref_h, ref_y = oracle.rollout(x, dt, A, B, C, h0=to_np(bank[1, 0]), want_y=True)
+    assert rel_err(to_np(h[0, 0, :64]), ref_h[:64]) < TOL_F32
+    assert rel_err(to_np(y[0, :, :64]), ref_y[:, :64]) < TOL_F32
