@@ -421,13 +421,15 @@ def measure_extensions(pg, synth, torch, dev, layer_in, off, T, n_chunks, index,
     sc = pg.scan_inputs(layer_in["x"], layer_in["dt"], layer_in["B"], A, a_kind=pg.PRECOG_A_COMPLEX)
     cst = torch.empty((n_chunks, 1, D, N, 2), dtype=torch.bfloat16, device=dev)
     ms = timed(lambda: pg.precog_encode_chunks(sc, off, T, states_out=cst), 3)
-    # SFU-bound: per state update one ex2 (32 per clock per SM on this GB300) and a sine
-    # and a cosine (16 each), measured with a throughput microbenchmark
+    # This A (real part -(n+1), imaginary part pi n in fp32) takes the power form: per state
+    # index one complex multiply of the power tree (4 FP32 lane operations) and the update
+    # h = alpha h + u B (6), i.e. 160 per channel-token on the FMA pipe (128 lane operations
+    # per clock per SM); the per-token sincosf and exponential are not counted.
     props = torch.cuda.get_device_properties(dev)
-    sfu_floor_ms = T * D * N * (1 / 32 + 2 / 16) / (props.multi_processor_count * 2.07e9) * 1e3
+    alu_floor_ms = T * D * N * 10 / (props.multi_processor_count * 128 * 2.07e9) * 1e3
     out["complex_A_encode"] = hbm_row(ms, in_bytes + cst.numel() * 2, tokens_per_s=T / (ms * 1e-3),
-                                      bound="alu (SFU: exp, sin, cos per state update)",
-                                      sfu_floor_ms_at_2070mhz=sfu_floor_ms, frac_sfu=sfu_floor_ms / ms)
+                                      bound="alu (FMA pipe: rotation tree and complex update)",
+                                      alu_floor_ms_at_2070mhz=alu_floor_ms, frac_alu=alu_floor_ms / ms)
     del cst
     # f1: top-3 retrieval over the 1M index and the composed 24-layer prefill
     M, dim = index.shape
