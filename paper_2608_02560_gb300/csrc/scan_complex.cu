@@ -1,9 +1,11 @@
 // The scan with the complex diagonal A that Eq. 1 prints (A_k = -softplus(a_k)
 // + i*pi*k, h in C^N): alpha = exp(dt * A) = e^(dt*A_re) (cos + i sin)(dt*A_im),
-// beta = B * x * dt real, y = Re(sum_n C_n h_n). Correctness-first: one thread
-// per channel with its 16 complex states in registers, inputs read straight
-// from global memory (coalesced across the channels of a block; B and C rows
-// are shared by the block and served from L1). One SFU exponential and one
+// beta = B * x * dt real, y = Re(sum_n C_n h_n). One thread per channel with its
+// 16 complex states in registers; blocks of 256 channels (128 with a readout,
+// whose update needs more registers) stage tiles of 16 tokens of their x and dt
+// row pieces and of the B (C) rows through a 3-stage shared-memory ring by TMA
+// bulk copies on mbarriers (one copy per tensor when the block spans the whole
+// row). Per-index form: one SFU exponential and one
 // sine/cosine pair per (token, channel, state index); the phase dt * A_im is
 // formed exactly as a two-float product (fma error term) and reduced to
 // [-pi, pi] by Cody-Waite with 2*pi split into two floats before the SFU
@@ -29,7 +31,6 @@ namespace {
 __device__ uint32_t g_scan_complex_status;
 
 constexpr int kN = 16;
-constexpr int kBlock = 128;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kInv2Pi = 0.15915494309189535f;
 constexpr float k2PiHi = 6.28318548202514648f;     // fp32 nearest to 2*pi
@@ -101,33 +102,43 @@ __device__ __forceinline__ void rotation(float th, float tl, float &c, float &s)
     s = fmaf(c0, tl, s0);
 }
 
-// One 16-value B or C row (32 or 64 bytes, 16-byte aligned), fetched raw with
-// vector loads one token ahead of its use; every thread of the block reads the
-// same row, so a warp issues one request per vector.
+// One 16-value B or C row of a staged tile, widened to fp32 (vector shared-memory loads;
+// every thread of the block reads the same row, a broadcast).
 template <typename TIn>
-struct RawRow {
-    static constexpr int kVec = static_cast<int>(kN * sizeof(TIn) / 16);
-    uint4 q[kVec];
-    __device__ __forceinline__ void load(const TIn *row) {
-        const uint4 *r = reinterpret_cast<const uint4 *>(row);
+__device__ __forceinline__ void widen_row(const TIn *row, float (&v)[kN]) {
+    constexpr int kVec = static_cast<int>(kN * sizeof(TIn) / 16);
+    const uint4 *r = reinterpret_cast<const uint4 *>(row);
 #pragma unroll
-        for (int i = 0; i < kVec; ++i) q[i] = __ldg(r + i);
-    }
-    __device__ __forceinline__ void widen(float (&v)[kN]) const {
+    for (int i = 0; i < kVec; ++i) {
+        const uint4 q = r[i];
+        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
 #pragma unroll
-        for (int i = 0; i < kVec; ++i) {
-            const uint32_t w[4] = {q[i].x, q[i].y, q[i].z, q[i].w};
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                if constexpr (std::is_same<TIn, float>::value) {
-                    v[4 * i + k] = __uint_as_float(w[k]);
-                } else {
-                    v[8 * i + 2 * k] = __uint_as_float(w[k] << 16);
-                    v[8 * i + 2 * k + 1] = __uint_as_float(w[k] & 0xffff0000u);
-                }
+        for (int k = 0; k < 4; ++k) {
+            if constexpr (std::is_same<TIn, float>::value) {
+                v[4 * i + k] = __uint_as_float(w[k]);
+            } else {
+                v[8 * i + 2 * k] = __uint_as_float(w[k] << 16);
+                v[8 * i + 2 * k + 1] = __uint_as_float(w[k] & 0xffff0000u);
             }
         }
     }
+}
+
+constexpr int kCT = 16;     // tokens per staged tile
+constexpr int kCS = 3;      // tiles in flight
+
+template <typename TIn, int CB>
+struct CTile {
+    TIn x[kCT * CB];        // row stride: the block's width W <= CB
+    TIn dt[kCT * CB];
+    TIn B[kCT * kN];
+    TIn C[kCT * kN];
+};
+
+template <typename TIn, int CB>
+struct CSmem {
+    uint64_t full[kCS];
+    alignas(128) CTile<TIn, CB> tile[kCS];
 };
 
 // Update forms of a block, from the structure of its A.
@@ -135,17 +146,27 @@ constexpr int kFormIndex = 0;     // one exponential and one sine/cosine per sta
 constexpr int kFormHarmonic = 1;  // A_im[n] = n A_im[1]: rotations from one sincosf
 constexpr int kFormPower = 2;     // and A_re[n] = (n+1) A_re[0]: alpha_n = m (m z)^n
 
+template <bool HAS_Y>
+constexpr int block_channels() { return HAS_Y ? 128 : 256; }
+
 template <typename TIn, bool HAS_Y, bool HAS_H0>
-__global__ void __launch_bounds__(kBlock)
+__global__ void __launch_bounds__(block_channels<HAS_Y>())
     scan_complex_kernel(const ScanParams p, const int cblocks) {
+    constexpr int CB = block_channels<HAS_Y>();
+    constexpr int SZ = static_cast<int>(sizeof(TIn));
+    extern __shared__ __align__(128) unsigned char smem_raw[];
+    CSmem<TIn, CB> &sm = *reinterpret_cast<CSmem<TIn, CB> *>(smem_raw);
     int64_t item = blockIdx.x;
     const int cb = static_cast<int>(item % cblocks);
     item /= cblocks;
     const int64_t chunk = item % p.n_chunks;
     const int layer = static_cast<int>(item / p.n_chunks);
-    const int d = cb * kBlock + threadIdx.x;
     const int D = p.D;
-    const bool live = d < D;
+    const int d0 = cb * CB;
+    const int W = D - d0 < CB ? D - d0 : CB;    // channels of this block (a multiple of 16 bytes)
+    const int tid = threadIdx.x;
+    const bool live = tid < W;
+    const int d = d0 + (live ? tid : 0);
     int64_t start, len;
     if (p.use_fixed) {
         start = chunk * p.fixed_len;
@@ -154,7 +175,7 @@ __global__ void __launch_bounds__(kBlock)
         start = p.offsets[chunk];
         const int64_t end = p.offsets[chunk + 1];
         if (start < 0 || end < start || end > p.T_tot) {
-            if (threadIdx.x == 0) atomicOr(&g_scan_complex_status, PRECOG_DEV_BAD_OFFSETS);
+            if (tid == 0) atomicOr(&g_scan_complex_status, PRECOG_DEV_BAD_OFFSETS);
             return;
         }
         len = end - start;
@@ -163,8 +184,43 @@ __global__ void __launch_bounds__(kBlock)
     const TIn *dtl = static_cast<const TIn *>(p.dt) + layer * p.ls_xd;
     const TIn *Bl = static_cast<const TIn *>(p.B) + layer * p.ls_bc;
     const TIn *Cl = HAS_Y ? static_cast<const TIn *>(p.C) + layer * p.ls_bc : nullptr;
-    const float2 *Al = reinterpret_cast<const float2 *>(p.A) +
-                       (static_cast<int64_t>(layer) * D + (live ? d : 0)) * kN;
+    const float2 *Al = reinterpret_cast<const float2 *>(p.A) + (static_cast<int64_t>(layer) * D + d) * kN;
+
+    // ---- staging ring: first tiles in flight while A and the initial state load ----
+    const int64_t ntiles = (len + kCT - 1) / kCT;
+    if (tid == 0) {
+        for (int s = 0; s < kCS; ++s) mbar_init(&sm.full[s], 1);
+        fence_barrier_init();
+    }
+    __syncthreads();
+    // warp 0: lane 0 states the tile's bytes, then the lanes copy it (one copy per tensor
+    // when the block spans the row, else one row piece per lane and tensor)
+    auto issue = [&](int64_t k) {
+        const int lane = tid & 31;
+        const int s = static_cast<int>(k % kCS);
+        CTile<TIn, CB> &tl = sm.tile[s];
+        const int64_t row0 = start + k * kCT;
+        const int ntok = static_cast<int>(len - k * kCT < kCT ? len - k * kCT : kCT);
+        const uint32_t rowb = static_cast<uint32_t>(W * SZ);
+        const uint32_t bcb = static_cast<uint32_t>(ntok * kN * SZ);
+        if (lane == 0) mbar_arrive_expect_tx(&sm.full[s], 2 * ntok * rowb + (HAS_Y ? 2 : 1) * bcb);
+        __syncwarp();
+        if (W == D) {
+            if (lane == 0) {
+                bulk_g2s(tl.x, xl + row0 * D, ntok * rowb, &sm.full[s]);
+                bulk_g2s(tl.dt, dtl + row0 * D, ntok * rowb, &sm.full[s]);
+            }
+        } else if (lane < ntok) {
+            bulk_g2s(tl.x + lane * W, xl + (row0 + lane) * D + d0, rowb, &sm.full[s]);
+            bulk_g2s(tl.dt + lane * W, dtl + (row0 + lane) * D + d0, rowb, &sm.full[s]);
+        }
+        if (lane == 0) {
+            bulk_g2s(tl.B, Bl + row0 * kN, bcb, &sm.full[s]);
+            if (HAS_Y) bulk_g2s(tl.C, Cl + row0 * kN, bcb, &sm.full[s]);
+        }
+    };
+    if (tid < 32)
+        for (int64_t k = 0; k < kCS && k < ntiles; ++k) issue(k);
 
     // state indices in pairs (2i, 2i+1): A_re * log2 e, A_im, -A_im, and the state
     constexpr int kP = kN / 2;
@@ -184,7 +240,6 @@ __global__ void __launch_bounds__(kBlock)
     // alpha) compounds over long memories past the 1e-5 agreement fp32 inputs are held to.
     const bool tree = !std::is_same<TIn, float>::value && __syncthreads_and(harmonic);
     const int form = tree ? (__syncthreads_and(power) ? kFormPower : kFormHarmonic) : kFormIndex;
-    if (!live) return;
     const float kre = re0 * kLog2e;
 
     float hr[kN], hi[kN];
@@ -196,113 +251,118 @@ __global__ void __launch_bounds__(kBlock)
     if constexpr (HAS_H0) {
         const int64_t row = p.idx ? p.idx[chunk] : chunk;
         if (row >= 0 && row < p.bank_entries) {
-            const int64_t off = ((row * p.L_bank + p.layer0 + layer) * static_cast<int64_t>(D) + d) * kN;
+            if (live) {
+                const int64_t off = ((row * p.L_bank + p.layer0 + layer) * static_cast<int64_t>(D) + d) * kN;
 #pragma unroll
-            for (int n = 0; n < kN; ++n) {
-                if (p.bank_dtype == PRECOG_F32) {
-                    const float2 v = reinterpret_cast<const float2 *>(p.bank)[off + n];
-                    hr[n] = v.x;
-                    hi[n] = v.y;
-                } else {
-                    const __nv_bfloat162 v = reinterpret_cast<const __nv_bfloat162 *>(p.bank)[off + n];
-                    hr[n] = __low2float(v);
-                    hi[n] = __high2float(v);
+                for (int n = 0; n < kN; ++n) {
+                    if (p.bank_dtype == PRECOG_F32) {
+                        const float2 v = reinterpret_cast<const float2 *>(p.bank)[off + n];
+                        hr[n] = v.x;
+                        hi[n] = v.y;
+                    } else {
+                        const __nv_bfloat162 v = reinterpret_cast<const __nv_bfloat162 *>(p.bank)[off + n];
+                        hr[n] = __low2float(v);
+                        hi[n] = __high2float(v);
+                    }
                 }
             }
-        } else if (!(p.idx && row == -1) && threadIdx.x == 0) {
+        } else if (!(p.idx && row == -1) && tid == 0) {
             atomicOr(&g_scan_complex_status, PRECOG_DEV_BAD_INDEX);
         }
     }
-    // token t+1's inputs are in flight while token t is computed
-    TIn nx{}, ndt{};
-    RawRow<TIn> nb{}, nc{};
-    const int64_t end = start + len;
-    if (len > 0) {
-        nx = xl[start * D + d];
-        ndt = dtl[start * D + d];
-        nb.load(Bl + start * kN);
-        if constexpr (HAS_Y) nc.load(Cl + start * kN);
-    }
-    for (int64_t t = start; t < end; ++t) {
-        const float xv = to_f32(nx);
-        const float dv = to_f32(ndt);
-        const float u = dv * xv;
-        float b[kN], cr[kN];
-        nb.widen(b);
-        if constexpr (HAS_Y) nc.widen(cr);
-        if (t + 1 < end) {
-            nx = xl[(t + 1) * D + d];
-            ndt = dtl[(t + 1) * D + d];
-            nb.load(Bl + (t + 1) * kN);
-            if constexpr (HAS_Y) nc.load(Cl + (t + 1) * kN);
-        }
-        const f2 dd = pack2(dv, dv), uu = pack2(u, u);
-        // alpha for the eight pairs of state indices: (re pair, im pair)
-        f2 are[kP], aim[kP];
-        if (form == kFormIndex) {
-#pragma unroll
-            for (int i = 0; i < kP; ++i) {
-                float e0, e1;
-                unpack2(mul2(dd, ar[i]), e0, e1);
-                const f2 mag = pack2(ex2(e0), ex2(e1));
-                const f2 th = mul2(dd, ai[i]);
-                const f2 tl = fma2(dd, ai[i], mul2(dd, nai[i]));   // exact error of the product
-                f2 sn, cs;
-                sincos_pair(th, tl, sn, cs);
-                are[i] = mul2(mag, cs);
-                aim[i] = mul2(mag, sn);
+
+    for (int64_t k = 0; k < ntiles; ++k) {
+        const int s = static_cast<int>(k % kCS);
+        const int ntok = static_cast<int>(len - k * kCT < kCT ? len - k * kCT : kCT);
+        const bool landed = mbar_wait(&sm.full[s], static_cast<uint32_t>((k / kCS) & 1));
+        if (!__syncthreads_and(landed)) {
+            // give up on this chunk: record it, let the copies already issued land, leave
+            if (tid == 0) {
+                atomicOr(&g_scan_complex_status, PRECOG_DEV_TIMEOUT);
+                for (int64_t k2 = k; k2 < k + kCS && k2 < ntiles; ++k2)
+                    mbar_wait(&sm.full[k2 % kCS], static_cast<uint32_t>((k2 / kCS) & 1));
             }
-        } else {
-            const float th = dv * a1;
-            float zr, zi;
-            rotation(th, fmaf(dv, a1, -th), zr, zi);
-            if (form == kFormPower) {
-                // alpha_n = m (m z)^n: pairs (alpha_2i, alpha_2i+1) = (m, m w) (w^2)^i, w = m z
-                const float m = ex2(dv * kre);
-                const float wr = m * zr, wi = m * zi;
-                are[0] = pack2(m, m * wr);
-                aim[0] = pack2(0.f, m * wi);
-                float w2r, w2i;
-                csquare(wr, wi, w2r, w2i);
-                power_tree(are, aim, w2r, w2i);
-            } else {
-                // rotations (z^2i, z^2i+1) = (1, z) (z^2)^i, then one magnitude per index
-                are[0] = pack2(1.f, zr);
-                aim[0] = pack2(0.f, zi);
-                float z2r, z2i;
-                csquare(zr, zi, z2r, z2i);
-                power_tree(are, aim, z2r, z2i);
+            return;
+        }
+        const CTile<TIn, CB> &tl = sm.tile[s];
+        for (int t = 0; t < ntok && live; ++t) {
+            const float xv = to_f32(tl.x[t * W + tid]);
+            const float dv = to_f32(tl.dt[t * W + tid]);
+            const float u = dv * xv;
+            float b[kN], cr[kN];
+            widen_row<TIn>(tl.B + t * kN, b);
+            if constexpr (HAS_Y) widen_row<TIn>(tl.C + t * kN, cr);
+            const f2 dd = pack2(dv, dv), uu = pack2(u, u);
+            // alpha for the eight pairs of state indices: (re pair, im pair)
+            f2 are[kP], aim[kP];
+            if (form == kFormIndex) {
 #pragma unroll
                 for (int i = 0; i < kP; ++i) {
                     float e0, e1;
                     unpack2(mul2(dd, ar[i]), e0, e1);
                     const f2 mag = pack2(ex2(e0), ex2(e1));
-                    are[i] = mul2(mag, are[i]);
-                    aim[i] = mul2(mag, aim[i]);
+                    const f2 th = mul2(dd, ai[i]);
+                    const f2 tl2 = fma2(dd, ai[i], mul2(dd, nai[i]));   // exact error of the product
+                    f2 sn, cs;
+                    sincos_pair(th, tl2, sn, cs);
+                    are[i] = mul2(mag, cs);
+                    aim[i] = mul2(mag, sn);
+                }
+            } else {
+                const float th = dv * a1;
+                float zr, zi;
+                rotation(th, fmaf(dv, a1, -th), zr, zi);
+                if (form == kFormPower) {
+                    // alpha_n = m (m z)^n: pairs (alpha_2i, alpha_2i+1) = (m, m w) (w^2)^i, w = m z
+                    const float m = ex2(dv * kre);
+                    const float wr = m * zr, wi = m * zi;
+                    are[0] = pack2(m, m * wr);
+                    aim[0] = pack2(0.f, m * wi);
+                    float w2r, w2i;
+                    csquare(wr, wi, w2r, w2i);
+                    power_tree(are, aim, w2r, w2i);
+                } else {
+                    // rotations (z^2i, z^2i+1) = (1, z) (z^2)^i, then one magnitude per index
+                    are[0] = pack2(1.f, zr);
+                    aim[0] = pack2(0.f, zi);
+                    float z2r, z2i;
+                    csquare(zr, zi, z2r, z2i);
+                    power_tree(are, aim, z2r, z2i);
+#pragma unroll
+                    for (int i = 0; i < kP; ++i) {
+                        float e0, e1;
+                        unpack2(mul2(dd, ar[i]), e0, e1);
+                        const f2 mag = pack2(ex2(e0), ex2(e1));
+                        are[i] = mul2(mag, are[i]);
+                        aim[i] = mul2(mag, aim[i]);
+                    }
                 }
             }
-        }
-        f2 y2 = pack2(0.f, 0.f);
+            f2 y2 = pack2(0.f, 0.f);
 #pragma unroll
-        for (int i = 0; i < kP; ++i) {
-            const f2 h_r = pack2(hr[2 * i], hr[2 * i + 1]), h_i = pack2(hi[2 * i], hi[2 * i + 1]);
-            const f2 nh_i = pack2(-hi[2 * i], -hi[2 * i + 1]);
-            const f2 nr = fma2(are[i], h_r, fma2(aim[i], nh_i, mul2(uu, pack2(b[2 * i], b[2 * i + 1]))));
-            const f2 ni = fma2(are[i], h_i, mul2(aim[i], h_r));
-            unpack2(nr, hr[2 * i], hr[2 * i + 1]);
-            unpack2(ni, hi[2 * i], hi[2 * i + 1]);
-            if constexpr (HAS_Y) y2 = fma2(pack2(cr[2 * i], cr[2 * i + 1]), nr, y2);
+            for (int i = 0; i < kP; ++i) {
+                const f2 h_r = pack2(hr[2 * i], hr[2 * i + 1]), h_i = pack2(hi[2 * i], hi[2 * i + 1]);
+                const f2 nh_i = pack2(-hi[2 * i], -hi[2 * i + 1]);
+                const f2 nr = fma2(are[i], h_r, fma2(aim[i], nh_i, mul2(uu, pack2(b[2 * i], b[2 * i + 1]))));
+                const f2 ni = fma2(are[i], h_i, mul2(aim[i], h_r));
+                unpack2(nr, hr[2 * i], hr[2 * i + 1]);
+                unpack2(ni, hi[2 * i], hi[2 * i + 1]);
+                if constexpr (HAS_Y) y2 = fma2(pack2(cr[2 * i], cr[2 * i + 1]), nr, y2);
+            }
+            if constexpr (HAS_Y) {
+                float y0, y1;
+                unpack2(y2, y0, y1);
+                const float y = y0 + y1;
+                const int64_t yo = (static_cast<int64_t>(layer) * p.T_tot + start + k * kCT + t) * D + d;
+                if (p.y_dtype == PRECOG_F32) static_cast<float *>(p.y)[yo] = y;
+                else static_cast<__nv_bfloat16 *>(p.y)[yo] = __float2bfloat16_rn(y);
+            }
         }
-        float y0, y1;
-        unpack2(y2, y0, y1);
-        const float y = y0 + y1;
-        if constexpr (HAS_Y) {
-            const int64_t yo = (static_cast<int64_t>(layer) * p.T_tot + t) * D + d;
-            if (p.y_dtype == PRECOG_F32) static_cast<float *>(p.y)[yo] = y;
-            else static_cast<__nv_bfloat16 *>(p.y)[yo] = __float2bfloat16_rn(y);
-        }
+        fence_proxy_async_smem();
+        __syncthreads();   // every thread is done with stage s
+        if (tid < 32 && k + kCS < ntiles) issue(k + kCS);
     }
-    if (p.states) {
+    if (p.states && live) {
         const int64_t off = ((chunk * p.L_out + p.layer0 + layer) * static_cast<int64_t>(D) + d) * kN;
 #pragma unroll
         for (int n = 0; n < kN; ++n) {
@@ -316,12 +376,18 @@ __global__ void __launch_bounds__(kBlock)
 
 template <typename TIn, bool HAS_Y, bool HAS_H0>
 cudaError_t launch_c(const ScanParams &p, cudaStream_t stream) {
-    const int cblocks = (p.D + kBlock - 1) / kBlock;
+    constexpr int CB = block_channels<HAS_Y>();
+    const int cblocks = (p.D + CB - 1) / CB;
     const int64_t items = static_cast<int64_t>(p.n_layers) * p.n_chunks * cblocks;
     if (items == 0) return cudaSuccess;
     if (items > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-    scan_complex_kernel<TIn, HAS_Y, HAS_H0><<<static_cast<unsigned>(items), kBlock, 0, stream>>>(p, cblocks);
-    cudaError_t e = cudaGetLastError();
+    const int smem = static_cast<int>(sizeof(CSmem<TIn, CB>));
+    static int smem_set = 0;
+    auto kern = scan_complex_kernel<TIn, HAS_Y, HAS_H0>;
+    cudaError_t e = ensure_smem(reinterpret_cast<const void *>(kern), &smem_set, smem);
+    if (e != cudaSuccess) return e;
+    kern<<<static_cast<unsigned>(items), CB, smem, stream>>>(p, cblocks);
+    e = cudaGetLastError();
     if (e == cudaSuccess) count_launches(1);
     return e;
 }
