@@ -139,12 +139,14 @@ def test_multi_layer_call_and_layer_offset(cuda_device):
             assert rel_err(got[c, 2 + l], ref[c]) < TOL_F32
 
 
-@pytest.mark.parametrize("D,y_mode", [(512, False), (1024, False), (1024, True), (768, True)])
+@pytest.mark.parametrize("D,y_mode", [(512, False), (1024, False), (768, False), (4096, False),
+                                      (1024, True), (768, True)])
 def test_multi_layer_sliced_channels(cuda_device, D, y_mode):
     """Rows wider than one CTA's channel slice (512 channels with the power-form A, 256
-    where 512 does not divide D), three layers in one call: each CTA stages its slice of
-    every x and dt row with one bulk copy per row; D = 512 stays one slice. Chunks end
-    inside and at the end of 16-row tiles. Every layer's states (and y) vs the oracle."""
+    where 512 does not divide D: 2, 3 and 8 slices here), three layers in one call: each
+    CTA stages its slice of every x and dt row with one bulk copy per row; D = 512 stays
+    one slice. Chunks (one of them empty) end inside and at the end of 16-row tiles.
+    Every layer's states (and y) vs the oracle."""
     import torch
     pg = _pg()
     d = cuda_device
