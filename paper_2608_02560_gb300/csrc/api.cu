@@ -2,7 +2,9 @@
 // kernels, status codes. Nothing here allocates device memory.
 #include <atomic>
 #include <cstdarg>
+#include <map>
 #include <mutex>
+#include <utility>
 #include <cstdio>
 #include <cstring>
 
@@ -95,6 +97,8 @@ precog::ScanParams base_params(const precog_scan_inputs *in, int64_t rows) {
 
 std::atomic<uint64_t> g_launches{0};
 std::mutex g_attr_mutex;
+// dynamic shared-memory limit already set, per (kernel, device): the attribute is per device
+std::map<std::pair<const void *, int>, int> g_smem_attr;
 
 }  // namespace
 
@@ -117,11 +121,15 @@ int device_sm_count() {
     return n;
 }
 
-cudaError_t ensure_smem(const void *kernel, int *cached_bytes, int bytes) {
+cudaError_t ensure_smem(const void *kernel, int bytes) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
     std::lock_guard<std::mutex> lock(g_attr_mutex);
-    if (*cached_bytes >= bytes) return cudaSuccess;
-    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-    if (e == cudaSuccess) *cached_bytes = bytes;
+    int &cached = g_smem_attr[std::make_pair(kernel, dev)];
+    if (cached >= bytes) return cudaSuccess;
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess) cached = bytes;
     return e;
 }
 

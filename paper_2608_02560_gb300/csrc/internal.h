@@ -64,9 +64,9 @@ bool encode_tiled_map(CUtensorMap *map, CUtensorMapDataType dtype, cuuint32_t ra
 // Kernel launches made by this library since the process started.
 void count_launches(uint64_t n);
 
-// Raise a kernel's dynamic shared-memory limit once per process (a host-side
+// Raise a kernel's dynamic shared-memory limit once per device (a host-side
 // attribute, not a stream operation, so later calls stay graph-capturable).
-cudaError_t ensure_smem(const void *kernel, int *cached_bytes, int bytes);
+cudaError_t ensure_smem(const void *kernel, int bytes);
 
 cudaError_t launch_scan(const ScanParams &p, cudaStream_t stream);
 

@@ -376,9 +376,8 @@ cudaError_t launch_tc(const RetrieveParams &p, int grid, cudaStream_t stream, ui
     if (!make_map(&tq, p.queries, p.n_queries, p.dim, bf16, a_rows) ||
         !make_map(&tk, p.index, p.M > 0 ? p.M : 1, p.dim, bf16, kBN))
         return cudaErrorInvalidValue;
-    static int smem_set = 0;
     const int smem = static_cast<int>(retrieve_tc_smem_bytes());
-    cudaError_t e = ensure_smem(reinterpret_cast<const void *>(retrieve_tc_kernel<LIST>), &smem_set, smem);
+    cudaError_t e = ensure_smem(reinterpret_cast<const void *>(retrieve_tc_kernel<LIST>), smem);
     if (e != cudaSuccess) return e;
     for (int q0 = 0; q0 < p.n_queries; q0 += 2 * kBM) {
         const int nq = p.n_queries - q0 < 2 * kBM ? p.n_queries - q0 : 2 * kBM;

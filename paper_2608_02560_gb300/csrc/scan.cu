@@ -767,8 +767,7 @@ cudaError_t launch_cfg(const ScanParams &p, cudaStream_t stream) {
     if (items == 0) return cudaSuccess;
     if (items > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
     auto kern = scan_kernel<C>;
-    static int smem_set = 0;
-    cudaError_t e = ensure_smem(reinterpret_cast<const void *>(kern), &smem_set, static_cast<int>(smem));
+    cudaError_t e = ensure_smem(reinterpret_cast<const void *>(kern), static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     kern<<<static_cast<unsigned>(items), DS / C::CPT, smem, stream>>>(p, DS, slices);
     e = cudaGetLastError();

@@ -382,9 +382,8 @@ cudaError_t launch_c(const ScanParams &p, cudaStream_t stream) {
     if (items == 0) return cudaSuccess;
     if (items > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
     const int smem = static_cast<int>(sizeof(CSmem<TIn, CB>));
-    static int smem_set = 0;
     auto kern = scan_complex_kernel<TIn, HAS_Y, HAS_H0>;
-    cudaError_t e = ensure_smem(reinterpret_cast<const void *>(kern), &smem_set, smem);
+    cudaError_t e = ensure_smem(reinterpret_cast<const void *>(kern), smem);
     if (e != cudaSuccess) return e;
     kern<<<static_cast<unsigned>(items), CB, smem, stream>>>(p, cblocks);
     e = cudaGetLastError();

@@ -691,14 +691,12 @@ cudaError_t launch_smc_consolidate(float *sem, int64_t n_slots, int64_t elems, c
         const int smem = static_cast<int>(sizeof(BulkSmem));
         cudaError_t e;
         if (states_dtype == PRECOG_BF16) {
-            static int attr_bf16 = 0;
-            e = ensure_smem(reinterpret_cast<const void *>(smc_consolidate_bulk_kernel<__nv_bfloat16>), &attr_bf16, smem);
+            e = ensure_smem(reinterpret_cast<const void *>(smc_consolidate_bulk_kernel<__nv_bfloat16>), smem);
             if (e != cudaSuccess) return e;
             smc_consolidate_bulk_kernel<__nv_bfloat16><<<static_cast<unsigned>(blocks2), kBulkThreads, smem, stream>>>(
                 sem, n_slots, elems, static_cast<const __nv_bfloat16 *>(states), slots, n, alpha, ntiles, per_cta);
         } else {
-            static int attr_f32 = 0;
-            e = ensure_smem(reinterpret_cast<const void *>(smc_consolidate_bulk_kernel<float>), &attr_f32, smem);
+            e = ensure_smem(reinterpret_cast<const void *>(smc_consolidate_bulk_kernel<float>), smem);
             if (e != cudaSuccess) return e;
             smc_consolidate_bulk_kernel<float><<<static_cast<unsigned>(blocks2), kBulkThreads, smem, stream>>>(
                 sem, n_slots, elems, static_cast<const float *>(states), slots, n, alpha, ntiles, per_cta);
