@@ -423,13 +423,28 @@ def measure_extensions(pg, synth, torch, dev, layer_in, off, T, n_chunks, index,
     ms = timed(lambda: pg.precog_encode_chunks(sc, off, T, states_out=cst), 3)
     # This A (real part -(n+1), imaginary part pi n in fp32) takes the power form: per state
     # index one complex multiply of the power tree (4 FP32 lane operations) and the update
-    # h = alpha h + u B (6), i.e. 160 per channel-token on the FMA pipe (128 lane operations
-    # per clock per SM); the per-token sincosf and exponential are not counted.
+    # h = alpha h + u B (5: u B, two for the real part, two for the imaginary part), i.e.
+    # 144 per channel-token on the FMA pipe (128 lane operations per clock per SM); the
+    # per-token sincosf and exponential are not counted.
     props = torch.cuda.get_device_properties(dev)
-    alu_floor_ms = T * D * N * 10 / (props.multi_processor_count * 128 * 2.07e9) * 1e3
+    alu_floor_ms = T * D * N * 9 / (props.multi_processor_count * 128 * 2.07e9) * 1e3
     out["complex_A_encode"] = hbm_row(ms, in_bytes + cst.numel() * 2, tokens_per_s=T / (ms * 1e-3),
                                       bound="alu (FMA pipe: rotation tree and complex update)",
                                       alu_floor_ms_at_2070mhz=alu_floor_ms, frac_alu=alu_floor_ms / ms)
+    # Eq. 1's own parameterisation: real part -softplus(a) per state index (no power
+    # structure), imaginary part pi*n: the harmonic form, one exponential per index plus
+    # the rotation tree: 12 FP32 lane operations per state index on the FMA pipe (the tree 4,
+    # the exponent 1, magnitude times rotation 2, the update 5)
+    g = torch.Generator(device=dev)
+    g.manual_seed(29)
+    re = -torch.nn.functional.softplus(torch.randn((D, N), generator=g, device=dev))
+    A = torch.complex(re, (math.pi * torch.arange(N, device=dev, dtype=torch.float32)).expand(D, N)).contiguous()
+    sc = pg.scan_inputs(layer_in["x"], layer_in["dt"], layer_in["B"], A, a_kind=pg.PRECOG_A_COMPLEX)
+    ms = timed(lambda: pg.precog_encode_chunks(sc, off, T, states_out=cst), 3)
+    alu_floor_ms = T * D * N * 12 / (props.multi_processor_count * 128 * 2.07e9) * 1e3
+    out["complex_A_encode_softplus_re"] = hbm_row(ms, in_bytes + cst.numel() * 2, tokens_per_s=T / (ms * 1e-3),
+                                                  bound="alu (FMA pipe; one SFU exponential per state index)",
+                                                  alu_floor_ms_at_2070mhz=alu_floor_ms, frac_alu=alu_floor_ms / ms)
     del cst
     # f1: top-3 retrieval over the 1M index and the composed 24-layer prefill
     M, dim = index.shape
