@@ -13,8 +13,8 @@
 //
 // Eq. 1's imaginary part is harmonic (A_im[n] = pi * n). When a block's A has
 // A_im[n] == n * A_im[1] exactly and its inputs are 16-bit, the 16 phase rotations of a token are the
-// powers z^n of one rotation z = e^(i dt A_im[1]) (one accurate sincosf per
-// token and channel, the exact product error folded in), formed by a complex
+// powers z^n of one rotation z = e^(i dt A_im[1]) (one reduced SFU sine and cosine
+// per token and channel, the exact product error folded in), formed by a complex
 // power tree of depth 3 on the FMA pipe; the magnitudes stay one exponential
 // per state index. When the real part is also of power form
 // (A_re[n] == (n+1) * A_re[0]), alpha_n = m * (m z)^n with m = e^(dt A_re[0])
@@ -94,12 +94,16 @@ __device__ __forceinline__ void power_tree(f2 (&pr)[8], f2 (&pi)[8], float z2r, 
     for (int j = 0; j < 4; ++j) cmul_pair(pr[j], pi[j], w8.r, w8.i, w8.ni, pr[4 + j], pi[4 + j]);
 }
 
-// e^(i (th + tl)) with th = dt * a the rounded product and tl its exact error.
+// e^(i (th + tl)) with th = dt * a the rounded product and tl its exact error: the phase
+// reduced to [-pi, pi] as in sincos_pair, then the SFU sine and cosine (absolute error
+// about 5e-7; the tree forms run only for 16-bit inputs, held to 2e-3).
 __device__ __forceinline__ void rotation(float th, float tl, float &c, float &s) {
-    float s0, c0;
-    sincosf(th, &s0, &c0);
-    c = fmaf(-s0, tl, c0);
-    s = fmaf(c0, tl, s0);
+    const float k = fmaf(fmaf(th, kInv2Pi, 12582912.f), 1.f, -12582912.f);
+    float r = fmaf(k, -k2PiHi, th);
+    r = fmaf(k, -k2PiLo, r);
+    r += tl;
+    asm("sin.approx.ftz.f32 %0, %1;" : "=f"(s) : "f"(r));
+    asm("cos.approx.ftz.f32 %0, %1;" : "=f"(c) : "f"(r));
 }
 
 // One 16-value B or C row of a staged tile, widened to fp32 (vector shared-memory loads;
