@@ -371,7 +371,8 @@ def run_case(args):
 # ------------------------------------------------------------------------------ extension rows
 
 
-def measure_extensions(pg, synth, torch, dev, layer_in, off, T, n_chunks, index, qbank, query_batch, hbm):
+def measure_extensions(pg, synth, torch, dev, layer_in, off, T, n_chunks, index, qbank, query_batch, hbm,
+                       call_in=None, layers_per_call=1):
     """Times the extension rows on the resident paper-shaped buffers (a few seconds):
     top-k retrieval and composed prefill (Sec. 4.4), K-dial trajectory capture (Sec. 5.2),
     the complex-A scan (Eq. 1's complex diagonal) and the SMC routing / EMA kernels (Sec. 5).
@@ -409,11 +410,15 @@ def measure_extensions(pg, synth, torch, dev, layer_in, off, T, n_chunks, index,
     lens = (off[1:] - off[:-1]).cpu().numpy()
     eo_np = np.concatenate([[0], np.cumsum((lens + stride - 1) // stride)]).astype(np.int64)
     eo = torch.from_numpy(eo_np).to(dev)
-    traj = torch.empty((int(eo_np[-1]), 1, D, N), dtype=torch.bfloat16, device=dev)
-    si = pg.scan_inputs(layer_in["x"], layer_in["dt"], layer_in["B"], layer_in["A"], a_kind=pg.PRECOG_A_POWER)
+    # as many layers per call as the encode (a launch's partial last wave is shared by them)
+    S = layers_per_call if call_in is not None else 1
+    traj = torch.empty((int(eo_np[-1]), S, D, N), dtype=torch.bfloat16, device=dev)
+    si = call_in if call_in is not None else pg.scan_inputs(layer_in["x"], layer_in["dt"], layer_in["B"],
+                                                            layer_in["A"], a_kind=pg.PRECOG_A_POWER)
     ms = timed(lambda: pg.precog_encode_trajectory(si, off, T, stride, eo, traj), 3)
-    out["trajectory_stride1000"] = hbm_row(ms, in_bytes + traj.numel() * 2, entries=int(eo_np[-1]),
-                                           tokens_per_s=T / (ms * 1e-3))
+    out["trajectory_stride1000"] = hbm_row(ms, S * in_bytes + traj.numel() * 2, entries=int(eo_np[-1]),
+                                           layers_per_call=S, ms_per_layer=ms / S,
+                                           tokens_per_s=S * T / (ms * 1e-3))
     del traj
     # f3: complex A, paper parameterisation (real part -(n+1), imaginary part pi*n)
     A = torch.complex(layer_in["A"], (math.pi * torch.arange(N, device=dev, dtype=torch.float32)).expand(D, N))
@@ -757,7 +762,7 @@ def main():
     extras = None
     if not args.no_extras:
         extras = measure_extensions(pg, synth, torch, dev, sets[0], off, T, shape.n_chunks, index, qbank,
-                                    query_batch, peaks()[0])
+                                    query_batch, peaks()[0], call_in=call_in, layers_per_call=S)
 
     st, bits = pg.precog_device_status()
     if st != 0:
