@@ -751,8 +751,10 @@ def main():
             with torch.cuda.graph(graph):
                 query_path(b)
             g50, _ = p50_p90(graph.replay, iters)
+            # the index sweep alone, at the measured copy bandwidth, bounds the latency below
+            floor_us = M * dim * index.element_size() / (peaks()[0] * 1e9) * 1e6
             latency[f"q{nq}"] = {"p50_us": p50, "p90_us": p90, "iters": iters,
-                                 "graph_p50_us": g50,
+                                 "graph_p50_us": g50, "index_sweep_floor_us": floor_us,
                                  "retrieved_planted": bool(torch.equal(b["idx"], b["rows"]))}
             del graph
             if b is not qb:
