@@ -420,6 +420,18 @@ def measure_extensions(pg, synth, torch, dev, layer_in, off, T, n_chunks, index,
                                            layers_per_call=S, ms_per_layer=ms / S,
                                            tokens_per_s=S * T / (ms * 1e-3))
     del traj
+    # a2 in its literal form: the same layer with A given as general (not stated as power
+    # form), one SFU exponential per (token, channel, state index): 16 per channel-token at
+    # 32 per clock per SM (measured) bound it
+    sg = pg.scan_inputs(layer_in["x"], layer_in["dt"], layer_in["B"], layer_in["A"], a_kind=pg.PRECOG_A_GENERAL)
+    gst = torch.empty((n_chunks, 1, D, N), dtype=torch.bfloat16, device=dev)
+    ms = timed(lambda: pg.precog_encode_chunks(sg, off, T, states_out=gst), 3)
+    props = torch.cuda.get_device_properties(dev)
+    sfu_floor_ms = T * D * N / (props.multi_processor_count * 32 * 2.07e9) * 1e3
+    out["encode_general_A"] = hbm_row(ms, in_bytes + gst.numel() * 2, tokens_per_s=T / (ms * 1e-3),
+                                      bound="alu (SFU: one exponential per state update)",
+                                      sfu_floor_ms_at_2070mhz=sfu_floor_ms, frac_sfu=sfu_floor_ms / ms)
+    del gst
     # f3: complex A, paper parameterisation (real part -(n+1), imaginary part pi*n)
     A = torch.complex(layer_in["A"], (math.pi * torch.arange(N, device=dev, dtype=torch.float32)).expand(D, N))
     A = A.contiguous()
