@@ -678,8 +678,9 @@ cudaError_t launch_smc_consolidate(float *sem, int64_t n_slots, int64_t elems, c
     if (blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
     const unsigned grid = static_cast<unsigned>(blocks);
     // Few slots: CTAs per (slot, element range). Each tile reads all n slot ids (from
-    // L2), n_slots / 512 of the state bytes for bf16 states, so it pays up to 256 slots.
-    // Whole 16-byte chunks per state row: the states stream through the TMA ring.
+    // L2): n_slots / 2048 of its state bytes with 16 KB ranges, so it pays up to 256
+    // slots. Rows of whole 16-byte chunks stream through the TMA ring; other rows take
+    // the register per-slot kernel (whose 2048-element ranges read n_slots / 512).
     const int64_t chunk = states_dtype == PRECOG_BF16 ? 8 : 4;
     if (n_slots >= 1 && n_slots <= 256 && elems % chunk == 0 && reinterpret_cast<uintptr_t>(slots) % 16 == 0) {
         const int64_t range = kStageBytes / (states_dtype == PRECOG_BF16 ? 2 : 4);
