@@ -5,20 +5,20 @@
 // whose update needs more registers) stage tiles of 16 tokens of their x and dt
 // row pieces and of the B (C) rows through a 3-stage shared-memory ring by TMA
 // bulk copies on mbarriers (one copy per tensor when the block spans the whole
-// row). Per-index form: one SFU exponential and one
-// sine/cosine pair per (token, channel, state index); the phase dt * A_im is
-// formed exactly as a two-float product (fma error term) and reduced to
-// [-pi, pi] by Cody-Waite with 2*pi split into two floats before the SFU
-// sine and cosine.
+// row). Per-index form: one SFU exponential and one sine/cosine pair per
+// (token, channel, state index); the phase dt * A_im is formed exactly as a
+// two-float product (fma error term) and reduced to [-pi, pi] by Cody-Waite with
+// 2*pi split into two floats before the SFU sine and cosine.
 //
 // Eq. 1's imaginary part is harmonic (A_im[n] = pi * n). When a block's A has
-// A_im[n] == n * A_im[1] exactly and its inputs are 16-bit, the 16 phase rotations of a token are the
-// powers z^n of one rotation z = e^(i dt A_im[1]) (one reduced SFU sine and cosine
-// per token and channel, the exact product error folded in), formed by a complex
-// power tree of depth 3 on the FMA pipe; the magnitudes stay one exponential
-// per state index. When the real part is also of power form
-// (A_re[n] == (n+1) * A_re[0]), alpha_n = m * (m z)^n with m = e^(dt A_re[0])
-// and the magnitudes ride in the same tree. Other A keep the per-index form.
+// A_im[n] == n * A_im[1] exactly and its inputs are 16-bit, the 16 phase
+// rotations of a token are the powers z^n of one rotation z = e^(i dt A_im[1])
+// (one reduced SFU sine and cosine per token and channel, the exact product error
+// folded in), formed by a complex power tree of depth 3 on the FMA pipe; the
+// magnitudes stay one exponential per state index (harmonic form). When the real
+// part is also of power form (A_re[n] == (n+1) * A_re[0]), alpha_n = m * (m z)^n
+// with m = e^(dt A_re[0]) and the magnitudes ride in the same tree (power form).
+// Other A, and fp32 inputs, keep the per-index form.
 #include <type_traits>
 
 #include "../../include/precog.h"
