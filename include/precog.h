@@ -282,6 +282,33 @@ precog_status precog_prefill_composed(const precog_scan_inputs *in, int32_t n_qu
                                       int32_t state_dtype, void *stream);
 
 /*
+ * precog_retrieve_keys -- precog_retrieve over one shard of an index whose rows are
+ * partitioned (e.g. across ranks): the shard holds rows row_offset .. row_offset+M-1
+ * of the whole index. For every query it writes one 64-bit key of its best row,
+ *   key = ((ordered bits of the fp32 score) << 32 | (2^32 - 1 - global row)) XOR 2^63,
+ * so that keys compare as signed int64 by score, then lower row ("no comparable row"
+ * is INT64_MIN). The signed maximum of the shards' keys (an all-reduce MAX over
+ * int64) is the key of the exact top-1 of the whole index, ties to the lowest global
+ * row, as precog_retrieve would return on the whole index; precog_decode_keys turns
+ * keys into rows and scores. This is the exchange step of row-sharded retrieval.
+ *   d_keys       device int64 [n_queries] (written)
+ *   row_offset   >= 0, with row_offset + M <= 2^32 - 1
+ * Other arguments and requirements as precog_retrieve (same workspace size).
+ */
+precog_status precog_retrieve_keys(const void *index, int32_t index_dtype, int64_t M, int32_t dim,
+                                   const void *queries, int32_t n_queries, int64_t row_offset,
+                                   int64_t *d_keys, void *workspace, size_t workspace_bytes,
+                                   void *stream);
+
+/*
+ * precog_decode_keys -- rows and scores of keys from precog_retrieve_keys (after
+ * combining shards): d_best_idx[q] = global row or -1, d_best_score[q] = score or NaN
+ * (d_best_score may be NULL).
+ */
+precog_status precog_decode_keys(const int64_t *d_keys, int32_t n_queries, int64_t *d_best_idx,
+                                 float *d_best_score, void *stream);
+
+/*
  * precog_smc_route -- two-level cluster routing of Structured Memory
  * Consolidation (Sec. 5.1, Eqs. smc-domain and smc-sub): for every embedding e
  * (a chunk's or an opening utterance's text embedding)

@@ -13,6 +13,7 @@ Functions carry the C names:
 * :func:`precog_retrieve`         -- exact top-1 retrieval (Sec. 4.2)
 * :func:`precog_prefill_from_state` -- injection (Eq. 2) + query prefill
 * :func:`precog_retrieve_topk`    -- top-k retrieval (Sec. 4.2 / 5.4)
+* :func:`precog_retrieve_keys`, :func:`precog_decode_keys` -- row-sharded retrieval
 * :func:`precog_prefill_composed` -- softmax-weighted top-k injection (Sec. 4.4) + prefill
 * :func:`precog_smc_route`, :func:`precog_smc_consolidate` -- SMC (Sec. 5)
 * :func:`precog_device_status`    -- device-side status word
@@ -67,6 +68,10 @@ def load_library(path: str = LIB_PATH):
                                          i32, vp, i32, vp]
     lib.precog_retrieve.restype = i32
     lib.precog_retrieve.argtypes = [vp, i32, i64, i32, vp, i32, vp, vp, vp, sz, vp]
+    lib.precog_retrieve_keys.restype = i32
+    lib.precog_retrieve_keys.argtypes = [vp, i32, i64, i32, vp, i32, i64, vp, vp, sz, vp]
+    lib.precog_decode_keys.restype = i32
+    lib.precog_decode_keys.argtypes = [vp, i32, vp, vp, vp]
     lib.precog_retrieve_workspace_size.restype = sz
     lib.precog_retrieve_workspace_size.argtypes = [i64, i32, i32]
     lib.precog_prefill_from_state.restype = i32
@@ -215,6 +220,29 @@ def precog_retrieve(index, queries, best_idx, best_score=None, workspace=None, s
         _ptr(index), _dtype_code(index), M, dim, _ptr(queries), Q, _ptr(best_idx),
         _ptr(best_score), _ptr(workspace), workspace.numel() * workspace.element_size(),
         _stream(stream)))
+
+
+def precog_retrieve_keys(index_shard, queries, row_offset: int, keys, workspace=None, stream=None):
+    """Best row of ``queries [Q, dim]`` in ``index_shard [M, dim]`` (rows ``row_offset ..``
+    of a row-partitioned index) as one signed-order int64 key per query in ``keys``; the
+    maximum over shards is the key of the whole index's top-1 (see precog.h)."""
+    import torch
+    lib = load_library()
+    M, dim = index_shard.shape
+    Q = queries.shape[0]
+    need = precog_retrieve_workspace_size(M, dim, Q)
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=queries.device)
+    _check(lib.precog_retrieve_keys(
+        _ptr(index_shard), _dtype_code(queries), M, dim, _ptr(queries), Q, int(row_offset), _ptr(keys),
+        _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def precog_decode_keys(keys, best_idx, best_score=None, stream=None):
+    """Rows (-1: none) and scores (NaN: none) of int64 keys from precog_retrieve_keys."""
+    lib = load_library()
+    _check(lib.precog_decode_keys(_ptr(keys), keys.shape[0], _ptr(best_idx), _ptr(best_score),
+                                  _stream(stream)))
 
 
 def precog_prefill_from_state(inputs: ScanInputs, n_queries: int, T_q: int, bank, idx=None,

@@ -398,6 +398,60 @@ precog_status precog_retrieve(const void *index, int32_t index_dtype, int64_t M,
     return ok();
 }
 
+precog_status precog_retrieve_keys(const void *index, int32_t index_dtype, int64_t M, int32_t dim,
+                                   const void *queries, int32_t n_queries, int64_t row_offset,
+                                   int64_t *d_keys, void *workspace, size_t workspace_bytes,
+                                   void *stream) {
+    const int sz = dtype_size(index_dtype);
+    if (sz == 0) return fail(PRECOG_ERR_UNSUPPORTED, "index_dtype must be F16, BF16 or F32");
+    if (M < 0) return fail(PRECOG_ERR_INVALID_ARG, "M must be >= 0");
+    if (M >= 0x7fffffffLL) return fail(PRECOG_ERR_UNSUPPORTED, "M must be below 2^31-1");
+    if (row_offset < 0 || row_offset + M > 0xffffffffLL)
+        return fail(PRECOG_ERR_INVALID_ARG, "need row_offset >= 0 and row_offset + M <= 2^32 - 1");
+    if (dim < 1) return fail(PRECOG_ERR_INVALID_ARG, "dim must be >= 1");
+    if ((static_cast<int64_t>(dim) * sz) % 16 != 0)
+        return fail(PRECOG_ERR_UNSUPPORTED, "dim*sizeof(dtype) must be a multiple of 16");
+    if (static_cast<int64_t>(dim) * sz > 8192)
+        return fail(PRECOG_ERR_UNSUPPORTED, "rows longer than 8 KiB (dim*sizeof(dtype)) are not implemented");
+    if (n_queries < 0) return fail(PRECOG_ERR_INVALID_ARG, "n_queries must be >= 0");
+    if (n_queries == 0) return ok();
+    if ((M > 0 && index == nullptr) || queries == nullptr || d_keys == nullptr)
+        return fail(PRECOG_ERR_INVALID_ARG, "index, queries and d_keys must be non-NULL");
+    if ((index && !aligned16(index)) || !aligned16(queries))
+        return fail(PRECOG_ERR_INVALID_ARG, "index and queries must be 16-byte aligned");
+    const size_t need = precog::retrieve_workspace_size(M, dim, n_queries);
+    if (workspace_bytes < need || (need > 0 && (workspace == nullptr || !aligned16(workspace))))
+        return fail(PRECOG_ERR_INVALID_ARG, "workspace too small or misaligned (%zu bytes needed)", need);
+    precog::RetrieveParams p;
+    p.index = index;
+    p.dtype = index_dtype;
+    p.M = M;
+    p.dim = dim;
+    p.queries = queries;
+    p.n_queries = n_queries;
+    p.best_idx = nullptr;
+    p.best_score = nullptr;
+    p.workspace = workspace;
+    p.workspace_bytes = workspace_bytes;
+    p.row_offset = row_offset;
+    p.keys_out = d_keys;
+    cudaError_t e = precog::launch_retrieve(p, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "retrieve launch");
+    return ok();
+}
+
+precog_status precog_decode_keys(const int64_t *d_keys, int32_t n_queries, int64_t *d_best_idx,
+                                 float *d_best_score, void *stream) {
+    if (n_queries < 0) return fail(PRECOG_ERR_INVALID_ARG, "n_queries must be >= 0");
+    if (n_queries == 0) return ok();
+    if (d_keys == nullptr || d_best_idx == nullptr)
+        return fail(PRECOG_ERR_INVALID_ARG, "d_keys and d_best_idx must be non-NULL");
+    cudaError_t e = precog::launch_decode_keys(d_keys, n_queries, d_best_idx, d_best_score,
+                                               static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "decode launch");
+    return ok();
+}
+
 precog_status precog_smc_route(const void *embeddings, int32_t dtype, int64_t n, int32_t dim,
                                const void *domain_protos, int32_t M, const void *sub_protos,
                                int32_t J_max, const int32_t *d_J, int32_t *d_domain, int32_t *d_sub,

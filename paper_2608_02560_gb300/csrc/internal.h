@@ -88,9 +88,15 @@ struct RetrieveParams {
     float *best_score;
     void *workspace;
     size_t workspace_bytes;
+    // shard mode (precog_retrieve_keys): rows are row_offset + local row, and the result
+    // is one signed-order key per query in keys_out instead of best_idx / best_score
+    int64_t row_offset = 0;
+    int64_t *keys_out = nullptr;
 };
 
 size_t retrieve_workspace_size(int64_t M, int32_t dim, int32_t n_queries);
+cudaError_t launch_decode_keys(const int64_t *keys, int32_t n, int64_t *best_idx, float *best_score,
+                               cudaStream_t stream);
 
 // Tensor-core path (retrieve_tc.cu): fp16/bf16 index, batches of queries.
 size_t retrieve_tc_smem_bytes();

@@ -158,11 +158,33 @@ __device__ __forceinline__ unsigned long long shfl_xor_u64(unsigned long long v,
     return (static_cast<unsigned long long>(hi) << 32) | lo;
 }
 
+// A shard's key with its row made global, in signed order: flipping the top bit
+// maps the unsigned key order onto int64 order, so keys of different shards combine
+// by a signed maximum (an all-reduce MAX over int64); "no row" becomes INT64_MIN.
+__device__ __forceinline__ int64_t global_key(unsigned long long k, int64_t row_offset) {
+    if (k != 0ull) {
+        const int64_t row = row_offset + static_cast<int64_t>(0xffffffffu - static_cast<uint32_t>(k & 0xffffffffu));
+        k = (k & 0xffffffff00000000ull) | static_cast<unsigned long long>(0xffffffffu - static_cast<uint32_t>(row));
+    }
+    return static_cast<int64_t>(k ^ 0x8000000000000000ull);
+}
+
+__device__ __forceinline__ void write_best(unsigned long long k, int64_t *best_idx, float *best_score, int q) {
+    if (k == 0ull) {
+        best_idx[q] = -1;
+        if (best_score) best_score[q] = __uint_as_float(0x7fc00000u);
+    } else {
+        best_idx[q] = static_cast<int64_t>(0xffffffffu - static_cast<uint32_t>(k & 0xffffffffu));
+        if (best_score) best_score[q] = unordered_float(static_cast<uint32_t>(k >> 32));
+    }
+}
+
 // One warp per query: each lane takes the maximum over a strided share of the
 // per-CTA keys (independent loads, so many are in flight), then a butterfly.
 __global__ void finalize_kernel(const unsigned long long *__restrict__ partial, int n_parts,
                                 int n_queries, int64_t *__restrict__ best_idx,
-                                float *__restrict__ best_score) {
+                                float *__restrict__ best_score, int64_t row_offset,
+                                int64_t *__restrict__ keys_out) {
     const int q = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
     if (q >= n_queries) return;
@@ -177,13 +199,16 @@ __global__ void finalize_kernel(const unsigned long long *__restrict__ partial, 
         k = v > k ? v : k;
     }
     if (lane != 0) return;
-    if (k == 0ull) {
-        best_idx[q] = -1;
-        if (best_score) best_score[q] = __uint_as_float(0x7fc00000u);
-    } else {
-        best_idx[q] = static_cast<int64_t>(0xffffffffu - static_cast<uint32_t>(k & 0xffffffffu));
-        if (best_score) best_score[q] = unordered_float(static_cast<uint32_t>(k >> 32));
-    }
+    if (keys_out) keys_out[q] = global_key(k, row_offset);
+    else write_best(k, best_idx, best_score, q);
+}
+
+// Signed-order keys (combined over shards) to rows and scores.
+__global__ void decode_keys_kernel(const int64_t *__restrict__ keys, int n, int64_t *__restrict__ best_idx,
+                                   float *__restrict__ best_score) {
+    const int q = blockIdx.x * blockDim.x + threadIdx.x;
+    if (q >= n) return;
+    write_best(static_cast<unsigned long long>(keys[q]) ^ 0x8000000000000000ull, best_idx, best_score, q);
 }
 
 // ---------------------------------------------------------------------------
@@ -433,11 +458,20 @@ cudaError_t launch_retrieve(const RetrieveParams &p, cudaStream_t stream) {
     if (e == cudaSuccess) {
         finalize_kernel<<<(p.n_queries + 3) / 4, 128, 0, stream>>>(
             static_cast<const unsigned long long *>(p.workspace), parts, p.n_queries, p.best_idx,
-            p.best_score);
+            p.best_score, p.row_offset, p.keys_out);
         e = cudaGetLastError();
         if (e == cudaSuccess) ++launches;
     }
     count_launches(launches);
+    return e;
+}
+
+cudaError_t launch_decode_keys(const int64_t *keys, int32_t n, int64_t *best_idx, float *best_score,
+                               cudaStream_t stream) {
+    if (n == 0) return cudaSuccess;
+    decode_keys_kernel<<<(n + 127) / 128, 128, 0, stream>>>(keys, n, best_idx, best_score);
+    cudaError_t e = cudaGetLastError();
+    if (e == cudaSuccess) count_launches(1);
     return e;
 }
 

@@ -60,3 +60,64 @@ def test_single_rank_helpers():
     assert bench.shard_seed(0) == 0 and bench.shard_seed(3) == 3000
     assert bench.reduce_max(4.5, 1, None) == 4.5
     assert bench.whole_job_rate(10, 1, 3, 2.0) == 15.0
+
+
+def _key(score, row):
+    """The documented shard key, written out independently: ordered score bits << 32 |
+    (2^32 - 1 - row), top bit flipped so that keys order as int64 (None: no row)."""
+    import numpy as np
+    if score is None:
+        return -(1 << 63)
+    u = int(np.array([score + 0.0], dtype=np.float32).view(np.uint32)[0])
+    ordered = (~u & 0xffffffff) if u & 0x80000000 else (u | 0x80000000)
+    k = ((ordered << 32) | (0xffffffff - row)) ^ (1 << 63)
+    return k - (1 << 64) if k >= (1 << 63) else k
+
+
+def _key_row(k):
+    if k == -(1 << 63):
+        return -1
+    return 0xffffffff - ((k + (1 << 64)) % (1 << 64) & 0xffffffff)
+
+
+# per query: (rank 0's best, rank 1's best) as (score, global row) or None
+_SHARD_BEST = [((0.9, 10), (0.8, 150)),        # the higher score wins
+               ((0.7, 20), (0.7, 120)),        # a tie: the lower global row
+               (None, (-0.5, 199)),            # one empty shard, a negative score
+               (None, None),                   # no comparable row anywhere
+               ((-0.0, 5), (0.0, 101))]        # -0 and +0 are the same score
+
+
+def _combine_main(rank, world, port, queue):
+    import torch
+    import torch.distributed as dist
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        from paper_2608_02560_gb300.distributed import combine_keys, shard_rows
+        keys = torch.tensor([_key(*b[rank]) if b[rank] else _key(None, 0) for b in _SHARD_BEST],
+                            dtype=torch.int64)
+        combine_keys(keys)
+        queue.put((rank, [_key_row(int(k)) for k in keys], shard_rows(200, world, rank)))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_gloo_ranks_combine_shard_keys():
+    """Row-sharded retrieval's exchange step: an all-reduce MAX over the shards' int64 keys
+    picks the higher score, then the lower global row, across ranks."""
+    mp = pytest.importorskip("torch.multiprocessing")
+    ctx = mp.get_context("spawn")
+    queue = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_combine_main, args=(r, 2, port, queue)) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(timeout=180)
+    assert all(p.exitcode == 0 for p in procs), [p.exitcode for p in procs]
+    res = sorted(queue.get(timeout=10) for _ in range(2))
+    (_, rows0, sh0), (_, rows1, sh1) = res
+    assert rows0 == rows1 == [10, 20, 199, -1, 5]
+    assert sh0 == (0, 100) and sh1 == (100, 100)
