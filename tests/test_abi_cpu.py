@@ -156,3 +156,21 @@ def test_selftest_rejects_bad_iteration_counts(lib):
     lib.precog_selftest_wait_timeout.restype = ctypes.c_int32
     assert lib.precog_selftest_wait_timeout(0, None) == 1
     assert lib.precog_selftest_wait_timeout((1 << 20) + 1, None) == 1
+
+
+def test_shard_key_calls_reject_bad_arguments(lib):
+    """Row-sharded retrieval: a negative row offset, an offset that pushes global rows past
+    2^32 - 1, missing key output and negative counts are argument errors returned before
+    any launch; zero queries is a no-op."""
+    f = lib.precog_retrieve_keys
+    ws = 1 << 20
+    assert f(FAKE, 2, 100, 768, FAKE, 1, -1, FAKE, FAKE, ws, None) == 1
+    assert f(FAKE, 2, 100, 768, FAKE, 1, (1 << 32) - 100, FAKE, FAKE, ws, None) == 1
+    assert f(FAKE, 2, 100, 768, FAKE, 1, 0, None, FAKE, ws, None) == 1
+    assert f(FAKE, 2, 100, 768, FAKE, 1, 0, FAKE, FAKE, 0, None) == 1          # no workspace
+    assert f(FAKE, 7, 100, 768, FAKE, 1, 0, FAKE, FAKE, ws, None) == 2          # dtype
+    assert f(FAKE, 2, 100, 768, FAKE, 0, 0, FAKE, FAKE, 0, None) == 0           # no queries
+    g = lib.precog_decode_keys
+    assert g(FAKE, -1, FAKE, FAKE, None) == 1
+    assert g(None, 3, FAKE, FAKE, None) == 1
+    assert g(FAKE, 0, FAKE, FAKE, None) == 0
