@@ -236,7 +236,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             int it = 0;
             for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
                 const int acc = it % nbuf;
-                // one lane waits, the warp follows its verdict (tcgen05.ld needs the whole warp)
+                // one lane waits, the warp follows its result (tcgen05.ld needs the whole warp)
                 bool ok = true;
                 if (lane == 0) ok = wait_or_abort(&sm.acc_full[acc], static_cast<uint32_t>(it / nbuf) & 1u, sm);
                 ok = __shfl_sync(0xffffffffu, ok, 0);
