@@ -2,8 +2,8 @@
 // + i*pi*k, h in C^N): alpha = exp(dt * A) = e^(dt*A_re) (cos + i sin)(dt*A_im),
 // beta = B * x * dt real, y = Re(sum_n C_n h_n). One thread per channel with its
 // 16 complex states in registers; blocks of 256 channels (128 with a readout,
-// whose update needs more registers) stage tiles of 16 tokens of their x and dt
-// row pieces and of the B (C) rows through a 3-stage shared-memory ring by TMA
+// whose update needs more registers) stage tiles of 32 tokens of their x and dt
+// row pieces and of the B (C) rows through a 2-stage shared-memory ring by TMA
 // bulk copies on mbarriers (one copy per tensor when the block spans the whole
 // row). Per-index form: one SFU exponential and one sine/cosine pair per
 // (token, channel, state index); the phase dt * A_im is formed exactly as a
@@ -128,8 +128,8 @@ __device__ __forceinline__ void widen_row(const TIn *row, float (&v)[kN]) {
     }
 }
 
-constexpr int kCT = 16;     // tokens per staged tile
-constexpr int kCS = 3;      // tiles in flight
+constexpr int kCT = 32;     // tokens per staged tile
+constexpr int kCS = 2;      // tiles in flight
 
 template <typename TIn, int CB>
 struct CTile {
