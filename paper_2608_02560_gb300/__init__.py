@@ -234,7 +234,7 @@ def precog_retrieve_keys(index_shard, queries, row_offset: int, keys, workspace=
     if workspace is None:
         workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=queries.device)
     _check(lib.precog_retrieve_keys(
-        _ptr(index_shard), _dtype_code(queries), M, dim, _ptr(queries), Q, int(row_offset), _ptr(keys),
+        _ptr(index_shard), _dtype_code(index_shard), M, dim, _ptr(queries), Q, int(row_offset), _ptr(keys),
         _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
