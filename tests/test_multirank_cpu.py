@@ -121,3 +121,18 @@ def test_two_gloo_ranks_combine_shard_keys():
     (_, rows0, sh0), (_, rows1, sh1) = res
     assert rows0 == rows1 == [10, 20, 199, -1, 5]
     assert sh0 == (0, 100) and sh1 == (100, 100)
+
+
+@pytest.mark.parametrize("M,world", [(0, 1), (0, 3), (1, 4), (7, 2), (10000, 3), (1_000_000, 8), (5, 8)])
+def test_shard_rows_tile_the_index(M, world):
+    """The ranks' row blocks are contiguous, in rank order, cover [0, M) exactly once and
+    differ in size by at most one row."""
+    from paper_2608_02560_gb300.distributed import shard_rows
+    blocks = [shard_rows(M, world, r) for r in range(world)]
+    pos = 0
+    for off, rows in blocks:
+        assert off == pos and rows >= 0
+        pos += rows
+    assert pos == M
+    sizes = [rows for _, rows in blocks]
+    assert max(sizes) - min(sizes) <= 1
