@@ -438,13 +438,13 @@ def measure_extensions(pg, synth, torch, dev, layer_in, off, T, n_chunks, index,
     sc = pg.scan_inputs(layer_in["x"], layer_in["dt"], layer_in["B"], A, a_kind=pg.PRECOG_A_COMPLEX)
     cst = torch.empty((n_chunks, 1, D, N, 2), dtype=torch.bfloat16, device=dev)
     ms = timed(lambda: pg.precog_encode_chunks(sc, off, T, states_out=cst), 3)
-    # This A (real part -(n+1), imaginary part pi n in fp32) takes the power form: per state
-    # index one complex multiply of the power tree (4 FP32 lane operations) and the update
-    # h = alpha h + u B (5: u B, two for the real part, two for the imaginary part), i.e.
-    # 144 per channel-token on the FMA pipe (128 lane operations per clock per SM); the
-    # per-token sincosf and exponential are not counted.
+    # This A (real part -(n+1), imaginary part pi n in fp32) takes the power form, and a
+    # capture without readout accumulates it rescaled: per state index one complex multiply
+    # of the power tree of the weights (4 FP32 lane operations) and two real FMAs adding
+    # w_n B_n to the rescaled state, i.e. 96 per channel-token on the FMA pipe (128 lane
+    # operations per clock per SM); the per-token exponent, phase and scale are not counted.
     props = torch.cuda.get_device_properties(dev)
-    alu_floor_ms = T * D * N * 9 / (props.multi_processor_count * 128 * 2.07e9) * 1e3
+    alu_floor_ms = T * D * N * 6 / (props.multi_processor_count * 128 * 2.07e9) * 1e3
     out["complex_A_encode"] = hbm_row(ms, in_bytes + cst.numel() * 2, tokens_per_s=T / (ms * 1e-3),
                                       bound="alu (FMA pipe: rotation tree and complex update)",
                                       alu_floor_ms_at_2070mhz=alu_floor_ms, frac_alu=alu_floor_ms / ms)

@@ -17,8 +17,10 @@
 // folded in), formed by a complex power tree of depth 3 on the FMA pipe; the
 // magnitudes stay one exponential per state index (harmonic form). When the real
 // part is also of power form (A_re[n] == (n+1) * A_re[0]), alpha_n = m * (m z)^n
-// with m = e^(dt A_re[0]) and the magnitudes ride in the same tree (power form).
-// Other A, and fp32 inputs, keep the per-index form.
+// with m = e^(dt A_re[0]) and the magnitudes ride in the same tree (power form); a
+// power-form capture without readout accumulates the state rescaled (one power tree
+// of the weights and two real FMAs per state index, see renormalise_c). Other A, and
+// fp32 inputs, keep the per-index form.
 #include <type_traits>
 
 #include "../../include/precog.h"
@@ -125,6 +127,111 @@ __device__ __forceinline__ void widen_row(const TIn *row, float (&v)[kN]) {
                 v[8 * i + 2 * k + 1] = __uint_as_float(w[k] & 0xffff0000u);
             }
         }
+    }
+}
+
+// ---- rescaled capture (power form, no readout) ----
+// With P_n(t) = prod of alpha_n over the tokens since the last renormalisation
+// = M^(n+1) Z^n (M = prod m, Z = prod z), the state is h_n = P_n G_n and a token adds
+//   G_n += u B_n P_n^-1 = u B_n E^(n+1) R^n,   E = M^-1 = 2^L, R = conj(Z) = e^(-i Phi),
+// L and Phi the running sums of dt * (-A_re[0] log2 e) and dt * A_im[1]: the weights
+// are one power tree of V = E R per token and channel and the update is two real FMAs
+// per state index (6 FP32 lane operations per index instead of the direct update's 9).
+// The block renormalises (h_n = P_n G_n, L = Phi = 0) when some lane's L would leave
+// [-kLmaxC, kLmaxC] (E^16 stays far inside fp32) and at least every kRenormTokens
+// tokens (the rounding of the running phase, which the tree multiplies by n, stays
+// below 64 roundings); a token whose own step leaves the window is applied directly.
+constexpr float kLmaxC = 6.0f;
+constexpr int kRenormTokens = 64;
+
+// Phi + th + tl reduced to [-pi, pi] (Cody-Waite with 2 pi split in two floats; the
+// rounding to an integer on the FMA pipe as in sincos_pair).
+__device__ __forceinline__ float wrap_phase(float phi, float th, float tl) {
+    const float a = (phi + th) + tl;
+    const float k = fmaf(fmaf(a, kInv2Pi, 12582912.f), 1.f, -12582912.f);
+    const float r = fmaf(k, -k2PiHi, a);
+    return fmaf(k, -k2PiLo, r);
+}
+
+// The sixteen alpha_n = m^(n+1) z^n of the power form as pairs (real, imaginary):
+// (alpha_2i, alpha_2i+1) = (m, m w) (w^2)^i with w = m z, m = 2^(dt A_re[0] log2 e),
+// z = e^(i dt A_im[1]).
+__device__ __forceinline__ void alpha_power(float dv, float a1, float kre, f2 (&are)[kN / 2],
+                                            f2 (&aim)[kN / 2]) {
+    const float th = dv * a1;
+    float zr, zi;
+    rotation(th, fmaf(dv, a1, -th), zr, zi);
+    const float m = ex2(dv * kre);
+    const float wr = m * zr, wi = m * zi;
+    are[0] = pack2(m, m * wr);
+    aim[0] = pack2(0.f, m * wi);
+    float w2r, w2i;
+    csquare(wr, wi, w2r, w2i);
+    power_tree(are, aim, w2r, w2i);
+}
+
+// h <- alpha h + u B for the sixteen complex states (held as real and imaginary arrays)
+__device__ __forceinline__ void update_direct(float (&hr)[kN], float (&hi)[kN], const f2 (&are)[kN / 2],
+                                              const f2 (&aim)[kN / 2], f2 uu, const float (&b)[kN]) {
+#pragma unroll
+    for (int i = 0; i < kN / 2; ++i) {
+        const f2 h_r = pack2(hr[2 * i], hr[2 * i + 1]), h_i = pack2(hi[2 * i], hi[2 * i + 1]);
+        const f2 nh_i = pack2(-hi[2 * i], -hi[2 * i + 1]);
+        const f2 nr = fma2(are[i], h_r, fma2(aim[i], nh_i, mul2(uu, pack2(b[2 * i], b[2 * i + 1]))));
+        const f2 ni = fma2(are[i], h_i, mul2(aim[i], h_r));
+        unpack2(nr, hr[2 * i], hr[2 * i + 1]);
+        unpack2(ni, hi[2 * i], hi[2 * i + 1]);
+    }
+}
+
+// h_n = M^(n+1) Z^n G_n with M = 2^-L, Z = e^(i phi); afterwards L = phi = 0
+__device__ __forceinline__ void renormalise_c(float (&hr)[kN], float (&hi)[kN], float &L, float &phi) {
+    const float M = ex2(-L);
+    float c, s;
+    asm("sin.approx.ftz.f32 %0, %1;" : "=f"(s) : "f"(phi));
+    asm("cos.approx.ftz.f32 %0, %1;" : "=f"(c) : "f"(phi));
+    const float vr = M * c, vi = M * s;
+    f2 are[kN / 2], aim[kN / 2];
+    are[0] = pack2(M, M * vr);
+    aim[0] = pack2(0.f, M * vi);
+    float v2r, v2i;
+    csquare(vr, vi, v2r, v2i);
+    power_tree(are, aim, v2r, v2i);
+#pragma unroll
+    for (int i = 0; i < kN / 2; ++i) {
+        const f2 g_r = pack2(hr[2 * i], hr[2 * i + 1]), g_i = pack2(hi[2 * i], hi[2 * i + 1]);
+        const f2 ng_i = pack2(-hi[2 * i], -hi[2 * i + 1]);
+        const f2 nr = fma2(are[i], g_r, mul2(aim[i], ng_i));
+        const f2 ni = fma2(are[i], g_i, mul2(aim[i], g_r));
+        unpack2(nr, hr[2 * i], hr[2 * i + 1]);
+        unpack2(ni, hi[2 * i], hi[2 * i + 1]);
+    }
+    L = 0.f;
+    phi = 0.f;
+}
+
+// G_n += u E^(n+1) R^n B_n with E = 2^L, R = e^(-i phi) (phi in [-pi, pi])
+__device__ __forceinline__ void accumulate_c(float (&hr)[kN], float (&hi)[kN], float u, float L, float phi,
+                                             const float (&b)[kN]) {
+    const float E = ex2(L);
+    float c, s;
+    asm("sin.approx.ftz.f32 %0, %1;" : "=f"(s) : "f"(phi));
+    asm("cos.approx.ftz.f32 %0, %1;" : "=f"(c) : "f"(phi));
+    const float vr = E * c, vi = -(E * s);
+    const float ue = u * E;
+    f2 wre[kN / 2], wim[kN / 2];
+    wre[0] = pack2(ue, ue * vr);
+    wim[0] = pack2(0.f, ue * vi);
+    float v2r, v2i;
+    csquare(vr, vi, v2r, v2i);
+    power_tree(wre, wim, v2r, v2i);
+#pragma unroll
+    for (int i = 0; i < kN / 2; ++i) {
+        const f2 bb = pack2(b[2 * i], b[2 * i + 1]);
+        const f2 g_r = fma2(wre[i], bb, pack2(hr[2 * i], hr[2 * i + 1]));
+        const f2 g_i = fma2(wim[i], bb, pack2(hi[2 * i], hi[2 * i + 1]));
+        unpack2(g_r, hr[2 * i], hr[2 * i + 1]);
+        unpack2(g_i, hi[2 * i], hi[2 * i + 1]);
     }
 }
 
@@ -275,21 +382,70 @@ __global__ void __launch_bounds__(block_channels<HAS_Y>())
         }
     }
 
-    for (int64_t k = 0; k < ntiles; ++k) {
-        const int s = static_cast<int>(k % kCS);
-        const int ntok = static_cast<int>(len - k * kCT < kCT ? len - k * kCT : kCT);
-        const bool landed = mbar_wait(&sm.full[s], static_cast<uint32_t>((k / kCS) & 1));
-        if (!__syncthreads_and(landed)) {
-            // give up on this chunk: record it, let the copies already issued land, leave
-            if (tid == 0) {
-                atomicOr(&g_scan_complex_status, PRECOG_DEV_TIMEOUT);
-                for (int64_t k2 = k; k2 < k + kCS && k2 < ntiles; ++k2)
-                    mbar_wait(&sm.full[k2 % kCS], static_cast<uint32_t>((k2 / kCS) & 1));
+    // Runs token(tile, t, k) for every token of the chunk, a staged tile at a time; false
+    // when a tile's wait hit its limit (recorded, and the copies already issued landed).
+    auto scan_tiles = [&](auto &&token) -> bool {
+        for (int64_t k = 0; k < ntiles; ++k) {
+            const int s = static_cast<int>(k % kCS);
+            const int ntok = static_cast<int>(len - k * kCT < kCT ? len - k * kCT : kCT);
+            const bool landed = mbar_wait(&sm.full[s], static_cast<uint32_t>((k / kCS) & 1));
+            if (!__syncthreads_and(landed)) {
+                if (tid == 0) {
+                    atomicOr(&g_scan_complex_status, PRECOG_DEV_TIMEOUT);
+                    for (int64_t k2 = k; k2 < k + kCS && k2 < ntiles; ++k2)
+                        mbar_wait(&sm.full[k2 % kCS], static_cast<uint32_t>((k2 / kCS) & 1));
+                }
+                return false;
             }
-            return;
+            const CTile<TIn, CB> &tl = sm.tile[s];
+            for (int t = 0; t < ntok && live; ++t) token(tl, t, k);
+            fence_proxy_async_smem();
+            __syncthreads();   // every thread is done with stage s
+            if (tid < 32 && k + kCS < ntiles) issue(k + kCS);
         }
-        const CTile<TIn, CB> &tl = sm.tile[s];
-        for (int t = 0; t < ntok && live; ++t) {
+        return true;
+    };
+
+    if (!HAS_Y && form == kFormPower) {
+        // rescaled capture: running exponent and phase, tokens since the last
+        // renormalisation (the same count on every lane), the live lanes of this warp
+        float Lc = 0.f, phc = 0.f;
+        int since = 0;
+        const unsigned lmask = __ballot_sync(0xffffffffu, live);
+        const bool done = scan_tiles([&](const CTile<TIn, CB> &tl, int t, int64_t) {
+            const float xv = to_f32(tl.x[t * W + tid]);
+            const float dv = to_f32(tl.dt[t * W + tid]);
+            const float u = dv * xv;
+            float b[kN];
+            widen_row<TIn>(tl.B + t * kN, b);
+            const f2 uu = pack2(u, u);
+            const float th = dv * a1, tle = fmaf(dv, a1, -th);
+            float Ln = fmaf(dv, -kre, Lc);
+            float ph = wrap_phase(phc, th, tle);
+            bool acc = true;
+            if (__any_sync(lmask, !(fabsf(Ln) <= kLmaxC) || since >= kRenormTokens)) {
+                renormalise_c(hr, hi, Lc, phc);
+                since = 0;
+                Ln = dv * -kre;
+                ph = wrap_phase(0.f, th, tle);
+                if (!(fabsf(Ln) <= kLmaxC)) {
+                    f2 are[kP], aim[kP];
+                    alpha_power(dv, a1, kre, are, aim);
+                    update_direct(hr, hi, are, aim, uu, b);
+                    Ln = 0.f;
+                    ph = 0.f;
+                    acc = false;
+                }
+            }
+            if (acc) accumulate_c(hr, hi, u, Ln, ph, b);
+            Lc = Ln;
+            phc = ph;
+            ++since;
+        });
+        if (!done) return;
+        if (live) renormalise_c(hr, hi, Lc, phc);
+    } else {
+        const bool done = scan_tiles([&](const CTile<TIn, CB> &tl, int t, int64_t k) {
             const float xv = to_f32(tl.x[t * W + tid]);
             const float dv = to_f32(tl.dt[t * W + tid]);
             const float u = dv * xv;
@@ -361,10 +517,8 @@ __global__ void __launch_bounds__(block_channels<HAS_Y>())
                 if (p.y_dtype == PRECOG_F32) static_cast<float *>(p.y)[yo] = y;
                 else static_cast<__nv_bfloat16 *>(p.y)[yo] = __float2bfloat16_rn(y);
             }
-        }
-        fence_proxy_async_smem();
-        __syncthreads();   // every thread is done with stage s
-        if (tid < 32 && k + kCS < ntiles) issue(k + kCS);
+        });
+        if (!done) return;
     }
     if (p.states && live) {
         const int64_t off = ((chunk * p.L_out + p.layer0 + layer) * static_cast<int64_t>(D) + d) * kN;

@@ -240,3 +240,50 @@ def test_complex_paper_shaped_launch_sampled(cuda_device):
         f = st[c, 0].float().cpu().numpy().astype(np.float64)
         assert rel_err_stored(f[..., 0], ref[0].real) < TOL_BF16, c
         assert rel_err_stored(f[..., 1], ref[0].imag) < TOL_BF16, c
+
+
+@pytest.mark.parametrize("regime", ["paper", "small_dt", "large_dt", "mixed_sign"])
+def test_complex_rescaled_capture_regimes(cuda_device, regime):
+    """Capture without readout for the power-form A accumulates rescaled: the block
+    renormalises when an exponent leaves its window and at least every 64 tokens, and a
+    token whose own step leaves the window is applied directly. Tiny steps (renormalised by
+    the token count, long memories), large steps (many tokens applied directly), steps of
+    both signs, and the state-only prefill from an injected state, against the oracle."""
+    import torch
+    pg = _pg()
+    d = cuda_device
+    D, N = 96, 16
+    offsets = np.array([0, 1, 1, 700, 2100, 2165], np.int64)
+    T = int(offsets[-1])
+    x, dt, _, B, C = synth.host_scan_inputs(T, D, N, seed=31)
+    rng = np.random.default_rng(32)
+    if regime == "small_dt":
+        dt = dt * 0.01
+    elif regime == "large_dt":
+        dt = dt + rng.choice([0.0, 9.0], size=dt.shape, p=[0.7, 0.3])
+    elif regime == "mixed_sign":
+        # steps of both signs, small enough that the states' growth stays inside fp32
+        dt = dt * rng.choice([-0.05, 0.05], size=dt.shape)
+    rnd = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.float32)).to(torch.bfloat16).float().numpy()
+    x, dt, B, C = rnd(x), rnd(dt), rnd(B), rnd(C)
+    A = _complex_A(D, N, 33, "power")
+    hs, _ = _encode(pg, d, x, dt, B, C, A, offsets, with_y=False, in_dtype=torch.bfloat16)
+    ref_h, _ = oracle.scan_complex(x, dt, A.real, A.imag, B, offsets)
+    assert _cplx_err(hs, ref_h) < TOL_BF16
+    assert np.all(hs[1] == 0)                         # the empty chunk keeps the zero state
+    # state-only prefill of 3 queries from injected states (rows 3, -1, 4)
+    Tq = 90
+    xq, dtq, _, Bq, Cq = synth.host_scan_inputs(3 * Tq, D, N, seed=34)
+    xq, dtq, Bq = rnd(xq), rnd(dtq), rnd(Bq)
+    bank = torch.from_numpy(hs.astype(np.complex64)).to(d).view(len(offsets) - 1, 1, D, N)
+    idx = torch.tensor([3, -1, 4], dtype=torch.int64, device=d)
+    h = torch.empty((3, 1, D, N), dtype=torch.complex64, device=d)
+    ins = pg.scan_inputs(_t(xq, d, torch.bfloat16), _t(dtq, d, torch.bfloat16), _t(Bq, d, torch.bfloat16),
+                         _t(A, d), a_kind=pg.PRECOG_A_COMPLEX)
+    pg.precog_prefill_from_state(ins, 3, Tq, bank, idx=idx, state_out=h)
+    assert pg.precog_device_status()[0] == 0
+    for q, row in enumerate([3, -1, 4]):
+        h0 = np.zeros((1, D, N), np.complex128) if row < 0 else hs[row].astype(np.complex64)[None]
+        sl = slice(q * Tq, (q + 1) * Tq)
+        ref, _ = oracle.scan_complex(xq[sl], dtq[sl], A.real, A.imag, Bq[sl], [0, Tq], h0=h0)
+        assert _cplx_err(h[q, 0].cpu().numpy(), ref[0]) < TOL_BF16
