@@ -250,6 +250,9 @@ template <typename TIn, int CB>
 struct CSmem {
     uint64_t full[kCS];
     alignas(128) CTile<TIn, CB> tile[kCS];
+    // the current tile's B and C rows widened to fp32 once per block (16-bit inputs)
+    alignas(16) float bw[kCT * kN];
+    alignas(16) float cw[kCT * kN];
 };
 
 // Update forms of a block, from the structure of its A.
@@ -382,6 +385,17 @@ __global__ void __launch_bounds__(block_channels<HAS_Y>())
         }
     }
 
+    // B and C rows of token t as fp32: the block's widened copy for 16-bit inputs
+    constexpr bool kWiden = !std::is_same<TIn, float>::value;
+    auto b_row = [&](const CTile<TIn, CB> &tl, int t) -> const float * {
+        if constexpr (kWiden) return sm.bw + t * kN;
+        else return reinterpret_cast<const float *>(tl.B) + t * kN;
+    };
+    auto c_row = [&](const CTile<TIn, CB> &tl, int t) -> const float * {
+        if constexpr (kWiden) return sm.cw + t * kN;
+        else return reinterpret_cast<const float *>(tl.C) + t * kN;
+    };
+
     // Runs token(tile, t, k) for every token of the chunk, a staged tile at a time; false
     // when a tile's wait hit its limit (recorded, and the copies already issued landed).
     auto scan_tiles = [&](auto &&token) -> bool {
@@ -389,6 +403,16 @@ __global__ void __launch_bounds__(block_channels<HAS_Y>())
             const int s = static_cast<int>(k % kCS);
             const int ntok = static_cast<int>(len - k * kCT < kCT ? len - k * kCT : kCT);
             const bool landed = mbar_wait(&sm.full[s], static_cast<uint32_t>((k / kCS) & 1));
+            if constexpr (kWiden) {
+                // every thread has seen the tile land; the barrier below publishes the rows
+                // (the previous tile's readers finished at the end of its iteration)
+                if (landed) {
+                    const CTile<TIn, CB> &tw = sm.tile[s];
+                    for (int i = tid; i < ntok * kN; i += CB) sm.bw[i] = to_f32(tw.B[i]);
+                    if (HAS_Y)
+                        for (int i = tid; i < ntok * kN; i += CB) sm.cw[i] = to_f32(tw.C[i]);
+                }
+            }
             if (!__syncthreads_and(landed)) {
                 if (tid == 0) {
                     atomicOr(&g_scan_complex_status, PRECOG_DEV_TIMEOUT);
@@ -417,7 +441,7 @@ __global__ void __launch_bounds__(block_channels<HAS_Y>())
             const float dv = to_f32(tl.dt[t * W + tid]);
             const float u = dv * xv;
             float b[kN];
-            widen_row<TIn>(tl.B + t * kN, b);
+            widen_row<float>(b_row(tl, t), b);
             const f2 uu = pack2(u, u);
             const float th = dv * a1, tle = fmaf(dv, a1, -th);
             float Ln = fmaf(dv, -kre, Lc);
@@ -450,8 +474,8 @@ __global__ void __launch_bounds__(block_channels<HAS_Y>())
             const float dv = to_f32(tl.dt[t * W + tid]);
             const float u = dv * xv;
             float b[kN], cr[kN];
-            widen_row<TIn>(tl.B + t * kN, b);
-            if constexpr (HAS_Y) widen_row<TIn>(tl.C + t * kN, cr);
+            widen_row<float>(b_row(tl, t), b);
+            if constexpr (HAS_Y) widen_row<float>(c_row(tl, t), cr);
             const f2 dd = pack2(dv, dv), uu = pack2(u, u);
             // alpha for the eight pairs of state indices: (re pair, im pair)
             f2 are[kP], aim[kP];
