@@ -18,8 +18,9 @@
 // magnitudes stay one exponential per state index (harmonic form). When the real
 // part is also of power form (A_re[n] == (n+1) * A_re[0]), alpha_n = m * (m z)^n
 // with m = e^(dt A_re[0]) and the magnitudes ride in the same tree (power form); a
-// power-form capture without readout accumulates the state rescaled (one power tree
-// of the weights and two real FMAs per state index, see renormalise_c). Other A, and
+// capture without readout accumulates the state rescaled (power form: one power tree
+// of the weights and two real FMAs per state index, see renormalise_c; harmonic form:
+// the rotation tree and one exponential per index, see renormalise_h). Other A, and
 // fp32 inputs, keep the per-index form.
 #include <type_traits>
 
@@ -230,6 +231,88 @@ __device__ __forceinline__ void accumulate_c(float (&hr)[kN], float (&hi)[kN], f
         const f2 bb = pack2(b[2 * i], b[2 * i + 1]);
         const f2 g_r = fma2(wre[i], bb, pack2(hr[2 * i], hr[2 * i + 1]));
         const f2 g_i = fma2(wim[i], bb, pack2(hi[2 * i], hi[2 * i + 1]));
+        unpack2(g_r, hr[2 * i], hr[2 * i + 1]);
+        unpack2(g_i, hi[2 * i], hi[2 * i + 1]);
+    }
+}
+
+// ---- rescaled capture, harmonic form (A_im[n] = n A_im[1], any A_re) ----
+// Here P_n = 2^(S c_n) Z^n with S the running sum of dt and c_n = A_re[n] log2 e, so a token
+// adds u B_n 2^(-S c_n) R^n: the rotations R^n from the power tree seeded with u, one SFU
+// exponential per state index for the magnitude, which multiplies B_n once for both the
+// real and the imaginary FMA (8 FP32 lane operations per index instead of the direct
+// update's 12). The weights' exponents -S c_n stay within [-kExpMaxC, kExpMaxC].
+constexpr float kExpMaxC = 96.0f;
+
+// pairs (s0 w^(2i), s0 w^(2i+1)) of the powers of w = (wr, wi), scaled by s0
+__device__ __forceinline__ void rot_tree(float s0, float wr, float wi, f2 (&pr)[kN / 2], f2 (&pi)[kN / 2]) {
+    pr[0] = pack2(s0, s0 * wr);
+    pi[0] = pack2(0.f, s0 * wi);
+    float w2r, w2i;
+    csquare(wr, wi, w2r, w2i);
+    power_tree(pr, pi, w2r, w2i);
+}
+
+// alpha_n = 2^(dt c_n) z^n of the harmonic form, z = e^(i dt A_im[1])
+__device__ __forceinline__ void alpha_harmonic(float dv, float a1, const f2 (&ar)[kN / 2], f2 (&are)[kN / 2],
+                                               f2 (&aim)[kN / 2]) {
+    const float th = dv * a1;
+    float zr, zi;
+    rotation(th, fmaf(dv, a1, -th), zr, zi);
+    rot_tree(1.f, zr, zi, are, aim);
+    const f2 dd = pack2(dv, dv);
+#pragma unroll
+    for (int i = 0; i < kN / 2; ++i) {
+        float e0, e1;
+        unpack2(mul2(dd, ar[i]), e0, e1);
+        const f2 mag = pack2(ex2(e0), ex2(e1));
+        are[i] = mul2(mag, are[i]);
+        aim[i] = mul2(mag, aim[i]);
+    }
+}
+
+// h_n = 2^(S c_n) Z^n G_n with Z = e^(i phi); afterwards S = phi = 0
+__device__ __forceinline__ void renormalise_h(float (&hr)[kN], float (&hi)[kN], const f2 (&ar)[kN / 2],
+                                              float &S, float &phi) {
+    float c, s;
+    asm("sin.approx.ftz.f32 %0, %1;" : "=f"(s) : "f"(phi));
+    asm("cos.approx.ftz.f32 %0, %1;" : "=f"(c) : "f"(phi));
+    f2 are[kN / 2], aim[kN / 2];
+    rot_tree(1.f, c, s, are, aim);
+    const f2 SS = pack2(S, S);
+#pragma unroll
+    for (int i = 0; i < kN / 2; ++i) {
+        float e0, e1;
+        unpack2(mul2(SS, ar[i]), e0, e1);
+        const f2 mag = pack2(ex2(e0), ex2(e1));
+        const f2 pr = mul2(mag, are[i]), pi = mul2(mag, aim[i]);
+        const f2 g_r = pack2(hr[2 * i], hr[2 * i + 1]), g_i = pack2(hi[2 * i], hi[2 * i + 1]);
+        const f2 ng_i = pack2(-hi[2 * i], -hi[2 * i + 1]);
+        const f2 nr = fma2(pr, g_r, mul2(pi, ng_i));
+        const f2 ni = fma2(pr, g_i, mul2(pi, g_r));
+        unpack2(nr, hr[2 * i], hr[2 * i + 1]);
+        unpack2(ni, hi[2 * i], hi[2 * i + 1]);
+    }
+    S = 0.f;
+    phi = 0.f;
+}
+
+// G_n += u 2^(-S c_n) R^n B_n with R = e^(-i phi) (phi in [-pi, pi])
+__device__ __forceinline__ void accumulate_h(float (&hr)[kN], float (&hi)[kN], const f2 (&ar)[kN / 2],
+                                             float u, float S, float phi, const float (&b)[kN]) {
+    float c, s;
+    asm("sin.approx.ftz.f32 %0, %1;" : "=f"(s) : "f"(phi));
+    asm("cos.approx.ftz.f32 %0, %1;" : "=f"(c) : "f"(phi));
+    f2 wre[kN / 2], wim[kN / 2];
+    rot_tree(u, c, -s, wre, wim);
+    const f2 nS = pack2(-S, -S);
+#pragma unroll
+    for (int i = 0; i < kN / 2; ++i) {
+        float e0, e1;
+        unpack2(mul2(nS, ar[i]), e0, e1);
+        const f2 mb = mul2(pack2(ex2(e0), ex2(e1)), pack2(b[2 * i], b[2 * i + 1]));
+        const f2 g_r = fma2(wre[i], mb, pack2(hr[2 * i], hr[2 * i + 1]));
+        const f2 g_i = fma2(wim[i], mb, pack2(hi[2 * i], hi[2 * i + 1]));
         unpack2(g_r, hr[2 * i], hr[2 * i + 1]);
         unpack2(g_i, hi[2 * i], hi[2 * i + 1]);
     }
@@ -468,6 +551,50 @@ __global__ void __launch_bounds__(block_channels<HAS_Y>())
         });
         if (!done) return;
         if (live) renormalise_c(hr, hi, Lc, phc);
+    } else if (!HAS_Y && form == kFormHarmonic) {
+        // rescaled capture, harmonic form: running sum of dt and phase; the window on the
+        // weights' exponents is |S| * max_n |c_n| <= kExpMaxC
+        float cmax = 0.f;
+#pragma unroll
+        for (int i = 0; i < kP; ++i) {
+            float c0, c1;
+            unpack2(ar[i], c0, c1);
+            cmax = fmaxf(cmax, fmaxf(fabsf(c0), fabsf(c1)));
+        }
+        float Sc = 0.f, phc = 0.f;
+        int since = 0;
+        const unsigned lmask = __ballot_sync(0xffffffffu, live);
+        const bool done = scan_tiles([&](const CTile<TIn, CB> &tl, int t, int64_t) {
+            const float xv = to_f32(tl.x[t * W + tid]);
+            const float dv = to_f32(tl.dt[t * W + tid]);
+            const float u = dv * xv;
+            float b[kN];
+            widen_row<float>(b_row(tl, t), b);
+            const float th = dv * a1, tle = fmaf(dv, a1, -th);
+            float Sn = Sc + dv;
+            float ph = wrap_phase(phc, th, tle);
+            bool acc = true;
+            if (__any_sync(lmask, !(fabsf(Sn) * cmax <= kExpMaxC) || since >= kRenormTokens)) {
+                renormalise_h(hr, hi, ar, Sc, phc);
+                since = 0;
+                Sn = dv;
+                ph = wrap_phase(0.f, th, tle);
+                if (!(fabsf(Sn) * cmax <= kExpMaxC)) {
+                    f2 are[kP], aim[kP];
+                    alpha_harmonic(dv, a1, ar, are, aim);
+                    update_direct(hr, hi, are, aim, pack2(u, u), b);
+                    Sn = 0.f;
+                    ph = 0.f;
+                    acc = false;
+                }
+            }
+            if (acc) accumulate_h(hr, hi, ar, u, Sn, ph, b);
+            Sc = Sn;
+            phc = ph;
+            ++since;
+        });
+        if (!done) return;
+        if (live) renormalise_h(hr, hi, ar, Sc, phc);
     } else {
         const bool done = scan_tiles([&](const CTile<TIn, CB> &tl, int t, int64_t k) {
             const float xv = to_f32(tl.x[t * W + tid]);
