@@ -449,16 +449,17 @@ def measure_extensions(pg, synth, torch, dev, layer_in, off, T, n_chunks, index,
                                       bound="alu (FMA pipe: rotation tree and complex update)",
                                       alu_floor_ms_at_2070mhz=alu_floor_ms, frac_alu=alu_floor_ms / ms)
     # Eq. 1's own parameterisation: real part -softplus(a) per state index (no power
-    # structure), imaginary part pi*n: the harmonic form, one exponential per index plus
-    # the rotation tree: 12 FP32 lane operations per state index on the FMA pipe (the tree 4,
-    # the exponent 1, magnitude times rotation 2, the update 5)
+    # structure), imaginary part pi*n: the harmonic form, accumulated rescaled in a capture:
+    # per state index the rotation tree 4 FP32 lane operations on the FMA pipe, the
+    # exponent's argument 1, the magnitude times B_n 1 and two FMAs into the rescaled state
+    # 2, i.e. 8 (the exponential itself runs on the SFU)
     g = torch.Generator(device=dev)
     g.manual_seed(29)
     re = -torch.nn.functional.softplus(torch.randn((D, N), generator=g, device=dev))
     A = torch.complex(re, (math.pi * torch.arange(N, device=dev, dtype=torch.float32)).expand(D, N)).contiguous()
     sc = pg.scan_inputs(layer_in["x"], layer_in["dt"], layer_in["B"], A, a_kind=pg.PRECOG_A_COMPLEX)
     ms = timed(lambda: pg.precog_encode_chunks(sc, off, T, states_out=cst), 3)
-    alu_floor_ms = T * D * N * 12 / (props.multi_processor_count * 128 * 2.07e9) * 1e3
+    alu_floor_ms = T * D * N * 8 / (props.multi_processor_count * 128 * 2.07e9) * 1e3
     out["complex_A_encode_softplus_re"] = hbm_row(ms, in_bytes + cst.numel() * 2, tokens_per_s=T / (ms * 1e-3),
                                                   bound="alu (FMA pipe; one SFU exponential per state index)",
                                                   alu_floor_ms_at_2070mhz=alu_floor_ms, frac_alu=alu_floor_ms / ms)
