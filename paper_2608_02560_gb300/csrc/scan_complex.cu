@@ -619,35 +619,10 @@ __global__ void __launch_bounds__(block_channels<HAS_Y>())
                     are[i] = mul2(mag, cs);
                     aim[i] = mul2(mag, sn);
                 }
+            } else if (form == kFormPower) {
+                alpha_power(dv, a1, kre, are, aim);
             } else {
-                const float th = dv * a1;
-                float zr, zi;
-                rotation(th, fmaf(dv, a1, -th), zr, zi);
-                if (form == kFormPower) {
-                    // alpha_n = m (m z)^n: pairs (alpha_2i, alpha_2i+1) = (m, m w) (w^2)^i, w = m z
-                    const float m = ex2(dv * kre);
-                    const float wr = m * zr, wi = m * zi;
-                    are[0] = pack2(m, m * wr);
-                    aim[0] = pack2(0.f, m * wi);
-                    float w2r, w2i;
-                    csquare(wr, wi, w2r, w2i);
-                    power_tree(are, aim, w2r, w2i);
-                } else {
-                    // rotations (z^2i, z^2i+1) = (1, z) (z^2)^i, then one magnitude per index
-                    are[0] = pack2(1.f, zr);
-                    aim[0] = pack2(0.f, zi);
-                    float z2r, z2i;
-                    csquare(zr, zi, z2r, z2i);
-                    power_tree(are, aim, z2r, z2i);
-#pragma unroll
-                    for (int i = 0; i < kP; ++i) {
-                        float e0, e1;
-                        unpack2(mul2(dd, ar[i]), e0, e1);
-                        const f2 mag = pack2(ex2(e0), ex2(e1));
-                        are[i] = mul2(mag, are[i]);
-                        aim[i] = mul2(mag, aim[i]);
-                    }
-                }
+                alpha_harmonic(dv, a1, ar, are, aim);
             }
             f2 y2 = pack2(0.f, 0.f);
 #pragma unroll
