@@ -20,6 +20,17 @@ MUTATIONS = {
     "readout_wrong_state": ("C[t * N + n] * h[n]", "C[t * N + n] * h[(n + 1) % N]"),
     "chunk_end_off_by_one": ("t < offsets[c + 1]; ++t", "t + 1 < offsets[c + 1]; ++t"),
     "ties_go_high": ("if (s > best)", "if (s >= best)"),
+    # the complex-A scan (Eq. 1's complex diagonal)
+    "complex_conjugate_rotation": ("A_re[d * N + n] + I * A_im[d * N + n]",
+                                   "A_re[d * N + n] - I * A_im[d * N + n]"),
+    "complex_parts_swapped": ("A_re[d * N + n] + I * A_im[d * N + n]",
+                              "A_im[d * N + n] + I * A_re[d * N + n]"),
+    "complex_rotation_dropped": ("cexp(dt_td * a)", "exp(dt_td * creal(a))"),
+    "complex_beta_imaginary": ("const double complex alpha = cexp(dt_td * a);\n"
+                               "                    const double beta = B[t * N + n] * x_td * dt_td;",
+                               "const double complex alpha = cexp(dt_td * a);\n"
+                               "                    const double complex beta = I * B[t * N + n] * x_td * dt_td;"),
+    "complex_readout_imaginary": ("C[t * N + n] * creal(h[n])", "C[t * N + n] * cimag(h[n])"),
 }
 
 PIN_TESTS = [
@@ -36,6 +47,8 @@ PIN_TESTS = [
     pins.test_retrieve_matches_numpy_argmax_first_occurrence,
     pins.test_retrieve_ties_nan_and_empty,
     pins.test_retrieve_planted_tiny_workload,
+    pins.test_complex_scan_real_special_case,
+    pins.test_complex_scan_theorem1_and_geometric_series,
 ]
 
 
@@ -57,7 +70,7 @@ def test_planted_mistake_is_caught(name, tmp_path, monkeypatch):
     so_path = _compile(src.replace(old, new), str(tmp_path), name)
     real = oracle._load()
     mutant = ctypes.CDLL(so_path)
-    for fn in ("oracle_scan", "oracle_retrieve"):
+    for fn in ("oracle_scan", "oracle_retrieve", "oracle_scan_complex"):
         getattr(mutant, fn).restype = getattr(real, fn).restype
         getattr(mutant, fn).argtypes = getattr(real, fn).argtypes
     monkeypatch.setattr(oracle, "_lib", mutant)
