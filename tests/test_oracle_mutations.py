@@ -20,6 +20,10 @@ MUTATIONS = {
     "readout_wrong_state": ("C[t * N + n] * h[n]", "C[t * N + n] * h[(n + 1) % N]"),
     "chunk_end_off_by_one": ("t < offsets[c + 1]; ++t", "t + 1 < offsets[c + 1]; ++t"),
     "ties_go_high": ("if (s > best)", "if (s >= best)"),
+    # the K-dial trajectory: the final state of a chunk whose length is not a multiple of
+    # the stride is not kept (fewer writes, never more)
+    "trajectory_final_state_dropped": ("if (step % stride == 0 || t + 1 == offsets[c + 1])",
+                                       "if (step % stride == 0)"),
     # the complex-A scan (Eq. 1's complex diagonal)
     "complex_conjugate_rotation": ("A_re[d * N + n] + I * A_im[d * N + n]",
                                    "A_re[d * N + n] - I * A_im[d * N + n]"),
@@ -47,6 +51,7 @@ PIN_TESTS = [
     pins.test_retrieve_matches_numpy_argmax_first_occurrence,
     pins.test_retrieve_ties_nan_and_empty,
     pins.test_retrieve_planted_tiny_workload,
+    lambda: pins.test_trajectory_is_prefix_rollouts(7),
     pins.test_complex_scan_real_special_case,
     pins.test_complex_scan_theorem1_and_geometric_series,
 ]
@@ -70,7 +75,7 @@ def test_planted_mistake_is_caught(name, tmp_path, monkeypatch):
     so_path = _compile(src.replace(old, new), str(tmp_path), name)
     real = oracle._load()
     mutant = ctypes.CDLL(so_path)
-    for fn in ("oracle_scan", "oracle_retrieve", "oracle_scan_complex"):
+    for fn in ("oracle_scan", "oracle_retrieve", "oracle_scan_complex", "oracle_trajectory"):
         getattr(mutant, fn).restype = getattr(real, fn).restype
         getattr(mutant, fn).argtypes = getattr(real, fn).argtypes
     monkeypatch.setattr(oracle, "_lib", mutant)
