@@ -86,3 +86,49 @@ def test_planted_mistake_is_caught(name, tmp_path, monkeypatch):
         except AssertionError:
             failures += 1
     assert failures > 0, f"no pin caught the planted mistake '{name}'"
+
+
+# Mistakes planted in the numpy routines of the oracle (top-k, composition, SMC).
+PY_SRC = os.path.join(os.path.dirname(oracle.__file__), "__init__.py")
+
+PY_MUTATIONS = {
+    "topk_ties_go_high": ("retrieve_topk", "        cand.sort()\n",
+                          "        cand.sort(key=lambda c: (c[0], -c[1]))\n"),
+    "topk_keeps_nan": ("retrieve_topk", "for i in range(M) if not np.isnan(S[q, i])]",
+                       "for i in range(M)]"),
+    "compose_temperature_inverted": ("compose", "z = s[valid] / temperature", "z = s[valid] * temperature"),
+    "compose_unnormalised": ("compose", "w = e / e.sum()", "w = e"),
+    "smc_route_ignores_J": ("smc_route", "retrieve(sub[m, : int(J[m])], emb[c:c + 1])",
+                            "retrieve(sub[m], emb[c:c + 1])"),
+    "smc_ema_weights_swapped": ("smc_consolidate", "out[slot] = (1.0 - alpha) * out[slot] + alpha * h[c]",
+                                "out[slot] = alpha * out[slot] + (1.0 - alpha) * h[c]"),
+}
+
+PY_PIN_TESTS = [
+    pins.test_topk_matches_numpy_stable_argsort,
+    pins.test_topk_nan_and_short_index,
+    pins.test_compose_softmax_weights,
+    pins.test_composition_commutes_with_the_scan,
+    pins.test_smc_route_two_levels,
+    pins.test_smc_consolidate_closed_form,
+]
+
+
+@pytest.mark.parametrize("name", sorted(PY_MUTATIONS))
+def test_planted_python_mistake_is_caught(name, monkeypatch):
+    import types
+    func, old, new = PY_MUTATIONS[name]
+    src = open(PY_SRC).read()
+    assert old in src, f"mutation anchor for {name} not found in the oracle source"
+    mutant = types.ModuleType("oracle_mutant")
+    mutant.__file__ = PY_SRC
+    exec(compile(src.replace(old, new), PY_SRC, "exec"), mutant.__dict__)
+    mutant._lib = oracle._load()                     # the unmutated C library
+    monkeypatch.setattr(oracle, func, getattr(mutant, func))
+    failures = 0
+    for pin in PY_PIN_TESTS:
+        try:
+            pin()
+        except AssertionError:
+            failures += 1
+    assert failures > 0, f"no pin caught the planted mistake '{name}'"

@@ -395,7 +395,7 @@ def test_smc_route_two_levels():
     P = np.array([[1.0, 0.0, 0.0], [0.0, 1.0, 0.0], [0.0, 0.0, 1.0]])
     Qs = np.zeros((3, 2, 3))
     Qs[0] = [[1.0, 1.0, 0.0], [1.0, -1.0, 0.0]]
-    Qs[1] = [[0.0, 1.0, 5.0], [0.0, 0.0, 0.0]]          # second entry unused (J[1] = 1)
+    Qs[1] = [[0.0, 1.0, 5.0], [0.0, 9.0, 9.0]]          # second entry unused (J[1] = 1), though it scores higher
     Qs[2] = [[0.0, 0.0, 1.0], [9.0, 9.0, 9.0]]
     J = [2, 1, 2]
     e = np.array([[0.9, -0.2, 0.1], [0.1, 0.8, 0.7], [0.2, 0.1, 0.95], [1.0, 1.0, 0.0]])
