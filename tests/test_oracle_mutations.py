@@ -20,6 +20,10 @@ MUTATIONS = {
     "readout_wrong_state": ("C[t * N + n] * h[n]", "C[t * N + n] * h[(n + 1) % N]"),
     "chunk_end_off_by_one": ("t < offsets[c + 1]; ++t", "t + 1 < offsets[c + 1]; ++t"),
     "ties_go_high": ("if (s > best)", "if (s >= best)"),
+    "initial_state_ignored": ("h[n] = (h0 != NULL) ? h0[(c * D + d) * N + n] : 0.0;", "h[n] = 0.0;"),
+    "first_key_skipped": ("for (int64_t i = 0; i < M; ++i) {", "for (int64_t i = 1; i < M; ++i) {"),
+    "dot_drops_last_dim": ("for (int64_t k = 0; k < dim; ++k)", "for (int64_t k = 0; k + 1 < dim; ++k)"),
+    "empty_index_scores_minus_inf": ("best_score[q] = (arg < 0) ? NAN : best;", "best_score[q] = best;"),
     # the K-dial trajectory: the final state of a chunk whose length is not a multiple of
     # the stride is not kept (fewer writes, never more)
     "trajectory_final_state_dropped": ("if (step % stride == 0 || t + 1 == offsets[c + 1])",
