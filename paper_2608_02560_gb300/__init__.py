@@ -101,6 +101,10 @@ def load_library(path: str = LIB_PATH):
     lib.precog_last_error.argtypes = []
     lib.precog_abi_version.restype = i32
     lib.precog_abi_version.argtypes = []
+    lib.precog_retrieve_noalloc.restype = i32
+    lib.precog_retrieve_noalloc.argtypes = [vp, i32, i64, i32, vp, i32, vp, vp, vp]
+    lib.precog_launch_count.restype = ctypes.c_uint64
+    lib.precog_launch_count.argtypes = []
     _lib = lib
     return lib
 
@@ -222,6 +226,16 @@ def precog_retrieve(index, queries, best_idx, best_score=None, workspace=None, s
         _stream(stream)))
 
 
+def precog_retrieve_noalloc(index, queries, best_idx, best_score=None, stream=None):
+    """precog_retrieve without a caller workspace: the partial keys go to a fixed device
+    array inside the library (at most about 430 queries per call; overlapping calls race)."""
+    lib = load_library()
+    M, dim = index.shape
+    _check(lib.precog_retrieve_noalloc(
+        _ptr(index), _dtype_code(index), M, dim, _ptr(queries), queries.shape[0], _ptr(best_idx),
+        _ptr(best_score), _stream(stream)))
+
+
 def precog_retrieve_keys(index_shard, queries, row_offset: int, keys, workspace=None, stream=None):
     """Best row of ``queries [Q, dim]`` in ``index_shard [M, dim]`` (rows ``row_offset ..``
     of a row-partitioned index) as one signed-order int64 key per query in ``keys``; the
@@ -322,3 +336,22 @@ def precog_device_status(stream=None):
     bits = ctypes.c_uint32(0)
     st = lib.precog_device_status(_stream(stream), ctypes.byref(bits))
     return st, bits.value
+
+
+def precog_status_string(status: int) -> str:
+    """The name of a precog_status code."""
+    return load_library().precog_status_string(int(status)).decode()
+
+
+def precog_last_error() -> str:
+    """The message of the last failed call on this host thread (empty if none)."""
+    return load_library().precog_last_error().decode()
+
+
+def precog_abi_version() -> int:
+    return int(load_library().precog_abi_version())
+
+
+def precog_launch_count() -> int:
+    """Kernels this process has launched through the library so far."""
+    return int(load_library().precog_launch_count())

@@ -174,3 +174,52 @@ def test_shard_key_calls_reject_bad_arguments(lib):
     assert g(FAKE, -1, FAKE, FAKE, None) == 1
     assert g(None, 3, FAKE, FAKE, None) == 1
     assert g(FAKE, 0, FAKE, FAKE, None) == 0
+
+
+def test_binding_has_every_declared_call():
+    """The Python binding carries every C-ABI entry point under the same name, and the
+    host-only ones answer without a GPU."""
+    import paper_2608_02560_gb300 as pg
+    for n in declared_functions():
+        assert callable(getattr(pg, n, None)), f"{n} has no same-named Python binding"
+    assert pg.precog_abi_version() == 1
+    assert pg.precog_status_string(1) == "PRECOG_ERR_INVALID_ARG"
+    assert pg.precog_launch_count() >= 0
+
+
+def test_extension_calls_reject_bad_arguments(lib):
+    """Top-k, trajectory, composition, SMC and no-workspace retrieval: invalid sizes,
+    counts and pointers return their status before any launch."""
+    import paper_2608_02560_gb300 as pg
+    ws = 1 << 20
+    t = lib.precog_retrieve_topk
+    assert t(FAKE, 2, 100, 768, FAKE, 1, 0, FAKE, FAKE, FAKE, ws, None) == 2     # k < 1
+    assert t(FAKE, 2, 100, 768, FAKE, 1, 9, FAKE, FAKE, FAKE, ws, None) == 2     # k > 8
+    assert t(FAKE, 2, 100, 768, FAKE, 1, 3, None, FAKE, FAKE, ws, None) == 1     # no d_idx
+    assert t(FAKE, 2, 100, 768, FAKE, 1, 3, FAKE, FAKE, FAKE, 0, None) == 1      # no workspace
+    assert t(FAKE, 2, 100, 768, FAKE, 0, 3, FAKE, FAKE, FAKE, 0, None) == 0      # no queries
+    s = _inputs(pg, a_kind=pg.PRECOG_A_POWER)
+    tr = lib.precog_encode_trajectory
+    assert tr(ctypes.byref(s), FAKE, 4, 64, 0, FAKE, FAKE, 0, 0, 1, None) == 1   # stride 0
+    assert tr(ctypes.byref(s), FAKE, 4, 64, 8, None, FAKE, 0, 0, 1, None) == 1   # no entry offsets
+    assert tr(ctypes.byref(s), FAKE, 4, 64, 8, FAKE, FAKE + 8, 0, 0, 1, None) == 1  # misaligned
+    assert tr(ctypes.byref(s), FAKE, 0, 64, 8, FAKE, FAKE, 0, 0, 1, None) == 0   # no chunks
+    c = lib.precog_prefill_composed
+    assert c(ctypes.byref(s), 2, 32, FAKE, 0, 10, 1, 0, 9, FAKE, FAKE, 1.0, FAKE, 0, None, 0, None) == 2
+    assert c(ctypes.byref(s), 2, 32, FAKE, 0, 10, 1, 0, 3, FAKE, None, 1.0, FAKE, 0, None, 0, None) == 1
+    assert c(ctypes.byref(s), 2, 32, FAKE, 0, 10, 1, 0, 3, FAKE, FAKE, 0.0, FAKE, 0, None, 0, None) == 1
+    assert c(ctypes.byref(s), 2, 32, FAKE, 0, 10, 1, 0, 3, FAKE, FAKE, 1.0, None, 0, None, 0, None) == 1
+    r = lib.precog_smc_route
+    assert r(FAKE, 7, 10, 64, FAKE, 4, FAKE, 8, FAKE, FAKE, FAKE, None, None) == 2   # dtype
+    assert r(FAKE, 2, 10, 0, FAKE, 4, FAKE, 8, FAKE, FAKE, FAKE, None, None) == 1    # dim 0
+    assert r(FAKE, 2, 10, 64, None, 4, FAKE, 8, FAKE, FAKE, FAKE, None, None) == 1   # no prototypes
+    assert r(FAKE, 2, 0, 64, FAKE, 4, FAKE, 8, FAKE, FAKE, FAKE, None, None) == 0    # nothing to route
+    k = lib.precog_smc_consolidate
+    assert k(FAKE, 4, 64, FAKE, 2, FAKE, 8, 0.5, None) == 2                          # fp16 states
+    assert k(FAKE, 4, 64, FAKE, 0, FAKE, 8, 0.0, None) == 1                          # alpha 0
+    assert k(FAKE, 4, 64, FAKE, 0, FAKE, 8, 1.5, None) == 1                          # alpha > 1
+    assert k(FAKE + 4, 4, 64, FAKE, 0, FAKE, 8, 0.5, None) == 1                      # misaligned
+    assert k(FAKE, 4, 64, FAKE, 0, FAKE, 0, 0.5, None) == 0                          # no deposits
+    n = lib.precog_retrieve_noalloc
+    assert n(FAKE, 2, 100, 768, FAKE, -1, FAKE, FAKE, None) == 1
+    assert n(FAKE, 2, -1, 768, FAKE, 1, FAKE, FAKE, None) == 1
