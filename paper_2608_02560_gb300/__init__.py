@@ -16,7 +16,9 @@ Functions carry the C names:
 * :func:`precog_retrieve_keys`, :func:`precog_decode_keys` -- row-sharded retrieval
 * :func:`precog_prefill_composed` -- softmax-weighted top-k injection (Sec. 4.4) + prefill
 * :func:`precog_smc_route`, :func:`precog_smc_consolidate` -- SMC (Sec. 5)
-* :func:`precog_device_status`    -- device-side status word
+* :func:`precog_retrieve_noalloc`  -- top-1 retrieval without a caller workspace
+* :func:`precog_device_status`    -- device-side status word; :func:`precog_status_string`,
+  :func:`precog_last_error`, :func:`precog_abi_version`, :func:`precog_launch_count`
 """
 from __future__ import annotations
 
