@@ -104,6 +104,8 @@ PY_MUTATIONS = {
     "compose_unnormalised": ("compose", "w = e / e.sum()", "w = e"),
     "smc_route_ignores_J": ("smc_route", "retrieve(sub[m, : int(J[m])], emb[c:c + 1])",
                             "retrieve(sub[m], emb[c:c + 1])"),
+    "smc_forgetting_slot_deposits": ("smc_consolidate", "        if slot < 0:\n            continue\n", ""),
+    "compose_missing_entries_weighted": ("compose", "valid = ~np.isnan(s)", "valid = np.ones(s.shape, dtype=bool)"),
     "smc_ema_weights_swapped": ("smc_consolidate", "out[slot] = (1.0 - alpha) * out[slot] + alpha * h[c]",
                                 "out[slot] = alpha * out[slot] + (1.0 - alpha) * h[c]"),
 }
