@@ -58,6 +58,15 @@ __device__ uint32_t g_scan_status;
 #ifndef PRECOG_RESCALED_GROUP
 #define PRECOG_RESCALED_GROUP 4
 #endif
+#ifndef PRECOG_RENORM_FLOOR
+#define PRECOG_RENORM_FLOOR 1
+#endif
+#ifndef PRECOG_FIXDS
+#define PRECOG_FIXDS 1
+#endif
+#ifndef PRECOG_E2_SFU
+#define PRECOG_E2_SFU 0
+#endif
 
 constexpr int kN = 16;          // state size (N) supported by the kernels
 constexpr int kMaxSlice = 256;  // channels per CTA at most (the default slice)
@@ -74,17 +83,21 @@ enum Mode { kGeneral = 0, kPower = 1 };
 constexpr int kTrajNone = 0, kTrajDirect = 1, kTrajRescaled = 2;
 
 template <typename TIn_, bool HAS_Y_, bool HAS_H0_, int MODE_, int CPT_, int TILE_, int STAGES_,
-          int MINB_, int TRAJ_ = kTrajNone, int MAXSLICE_ = kMaxSlice>
+          int MINB_, int TRAJ_ = kTrajNone, int MAXSLICE_ = kMaxSlice, int FIXDS_ = 0>
 struct Cfg {
     using TIn = TIn_;
+    // Channel slice known at compile time (0: a launch argument). A constant slice turns
+    // the shared-memory row offsets of the time loop into immediates.
+    static constexpr int FIXDS = FIXDS_;
     // Widest channel slice of one CTA. Each CTA stages its slice of every token row; a
     // slice narrower than the row turns the row into separate pieces, and HBM serves
     // short scattered pieces far below its streaming rate, so rows up to 512 channels
     // stay whole. MINB counts resident CTAs of kMaxSlice channels (the register budget
     // per thread), whatever the slice.
     static constexpr int MAXSLICE = MAXSLICE_;
-    static constexpr int LB_THREADS = MAXSLICE_ / CPT_;
-    static constexpr int LB_BLOCKS = MINB_ * kMaxSlice / MAXSLICE_ > 0 ? MINB_ * kMaxSlice / MAXSLICE_ : 1;
+    static constexpr int LB_SLICE = FIXDS_ ? FIXDS_ : MAXSLICE_;
+    static constexpr int LB_THREADS = LB_SLICE / CPT_;
+    static constexpr int LB_BLOCKS = MINB_ * kMaxSlice / LB_SLICE > 0 ? MINB_ * kMaxSlice / LB_SLICE : 1;
     static constexpr bool HAS_Y = HAS_Y_, HAS_H0 = HAS_H0_;
     // keep every stride-th state (K-dial, Sec. 5.2), with the direct or the rescaled update
     static constexpr int TRAJ = TRAJ_;
@@ -351,7 +364,13 @@ __device__ __forceinline__ void renormalise(f2 (&g)[8], float &L) {
 __device__ __forceinline__ void accumulate(f2 (&g)[8], const f2 (&b)[8], float u, float Ln) {
     const float E = ex2(Ln);
     const float w0 = u * E;
+#if PRECOG_E2_SFU
+    // 2^(2 Ln) from the SFU: doubling Ln exactly by an exponent-field add (|Ln| <= kLmax
+    // here, or 0; a zero becomes 2^-126, whose exponential is 1 as well)
+    const float E2 = ex2(__int_as_float(__float_as_int(Ln) + 0x00800000));
+#else
     const float E2 = E * E;
+#endif
     f2 w = pack2(w0, w0 * E);
     const f2 ee = pack2(E2, E2);
     g[0] = fma2(w, b[0], g[0]);
@@ -399,12 +418,39 @@ __device__ __forceinline__ void token_checked(f2 (&g)[CPT][8], float (&L)[CPT],
     }
 }
 
+// Moves the frame of G to the bottom of the window: h_n = G_n E^-(n+1) is re-expressed
+// with L = -kLmax, G_n <- G_n 2^-((n+1)(L + kLmax)). With dt >= 0 the exponent then
+// climbs through the whole window [-kLmax, kLmax] before the next renormalisation,
+// twice as many tokens as a restart from L = 0. The factor of states 8..15 can fall
+// below the fp32 range (s = L + kLmax <= 2 kLmax), so they take it in two multiplies,
+// 2^-8s first; every factor and every intermediate stays within 2^(+-16 kLmax).
+__device__ __forceinline__ void renorm_floor(f2 (&g)[8], float &L) {
+    const float r = ex2(-(L + kLmax));
+    const float r2 = r * r;
+    f2 p[4];
+    p[0] = pack2(r, r2);
+    const f2 rr = pack2(r2, r2);
+#pragma unroll
+    for (int i = 1; i < 4; ++i) p[i] = mul2(p[i - 1], rr);
+    float r7, r8;
+    unpack2(p[3], r7, r8);
+    const f2 q = pack2(r8, r8);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) g[i] = mul2(g[i], p[i]);
+#pragma unroll
+    for (int i = 4; i < 8; ++i) g[i] = mul2(mul2(g[i], q), p[i - 4]);
+    L = -kLmax;
+}
+
 // Tokens go in groups of kGroup. The group's exponents are summed first (one
 // serial FMA per token and channel). With dt >= 0 they only grow, so checking
-// the group's last exponent covers every token in it; a negative dt anywhere
-// in the group (seen from the sign bits) sends the group through the per-token
-// check. One warp vote per group; the fast path then carries no branch, so the
-// power chains of the group's tokens can interleave.
+// the group's last exponent covers every token in it. One warp vote per group;
+// the fast path then carries no branch, so the power chains of the group's
+// tokens can interleave. When some lane's exponent would leave the window, the
+// warp renormalises every channel to the bottom of the window before the group
+// and takes the fast path all the same; only a negative dt anywhere in the group
+// (seen from the sign bits) or a group whose own exponent increment exceeds the
+// whole window goes through the per-token check.
 constexpr int kGroup = PRECOG_RESCALED_GROUP;
 
 template <class C>
@@ -427,10 +473,30 @@ __device__ __forceinline__ void scan_tile_rescaled(const unsigned char *st, cons
 #pragma unroll
             for (int j = 0; j < CPT; ++j) Lk[k][j] = fmaf(dvk[k][j], kk[j], k ? Lk[k - 1][j] : L[j]);
         }
-        bool need = neg != 0;
+        bool up = false;
 #pragma unroll
-        for (int j = 0; j < CPT; ++j) need |= !(fabsf(Lk[kGroup - 1][j]) <= kLmax);
-        if (__any_sync(wmask, need)) {
+        for (int j = 0; j < CPT; ++j) up |= !(Lk[kGroup - 1][j] <= kLmax);
+        bool slow = false;
+        if (__any_sync(wmask, up || neg != 0)) {
+#if PRECOG_RENORM_FLOOR
+            slow = __any_sync(wmask, neg != 0);
+            if (!slow) {
+#pragma unroll
+                for (int j = 0; j < CPT; ++j) renorm_floor(g[j], L[j]);
+                bool up2 = false;
+#pragma unroll
+                for (int k = 0; k < kGroup; ++k)
+#pragma unroll
+                    for (int j = 0; j < CPT; ++j) Lk[k][j] = fmaf(dvk[k][j], kk[j], k ? Lk[k - 1][j] : L[j]);
+#pragma unroll
+                for (int j = 0; j < CPT; ++j) up2 |= !(Lk[kGroup - 1][j] <= kLmax);
+                slow = __any_sync(wmask, up2);
+            }
+#else
+            slow = true;
+#endif
+        }
+        if (slow) {
             // unrolled so that dvk stays in registers (no dynamic indexing)
 #pragma unroll
             for (int k = 0; k < kGroup; ++k) {
@@ -470,8 +536,9 @@ __device__ __forceinline__ void scan_tile_rescaled(const unsigned char *st, cons
 // ---------------------------------------------------------------------------
 template <class C>
 __global__ void __launch_bounds__(C::LB_THREADS, C::LB_BLOCKS)
-    scan_kernel(const ScanParams p, const int DS, const int slices) {
+    scan_kernel(const ScanParams p, const int DS_arg, const int slices) {
     using TIn = typename C::TIn;
+    const int DS = C::FIXDS ? C::FIXDS : DS_arg;
     constexpr int CPT = C::CPT, TILE = C::TILE, STAGES = C::STAGES, SZ = C::SZ;
     extern __shared__ __align__(128) unsigned char smem[];
     uint64_t *full = reinterpret_cast<uint64_t *>(smem);
@@ -759,7 +826,7 @@ bool few_items(const ScanParams &p) {
 template <class C>
 cudaError_t launch_cfg(const ScanParams &p, cudaStream_t stream) {
     const int DS = pick_slice(p.D, C::SZ, C::CPT, C::MAXSLICE);
-    if (DS == 0) return cudaErrorInvalidValue;
+    if (DS == 0 || (C::FIXDS && DS != C::FIXDS)) return cudaErrorInvalidValue;
     const int slices = p.D / DS;
     const StageLayout lay = stage_layout(C::TILE, DS, C::SZ, C::HAS_Y, C::CONV);
     const size_t smem = kBarBytes + static_cast<size_t>(C::STAGES) * lay.bytes;
@@ -790,6 +857,15 @@ cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
         else
             return launch_cfg<Cfg<TIn, false, false, MODE, 2, 16, 4, 3, kTrajDirect>>(p, stream);
     } else if constexpr (MODE == kPower && !HAS_Y) {
+#if PRECOG_FIXDS
+        // the corpus encode of 256-channel rows (the paper's layer width) gets a slice fixed
+        // at compile time
+        if constexpr (!HAS_H0 && !std::is_same<TIn, float>::value)
+            if (pick_slice(p.D, sizeof(TIn), PRECOG_RESCALED_CPT, kWideSlice) == 256)
+                return launch_cfg<Cfg<TIn, false, false, MODE, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
+                                      PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB, kTrajNone, kWideSlice,
+                                      256>>(p, stream);
+#endif
         return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
                               PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB, kTrajNone, kWideSlice>>(p, stream);
     } else {
