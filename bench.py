@@ -63,6 +63,8 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-latency", action="store_true")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the single-layer wide and the ragged large-scale encode measurements")
     ap.add_argument("--no-extras", action="store_true",
                     help="skip the measurements of the extension rows (top-k, trajectory, complex A, SMC)")
     ap.add_argument("--case", choices=["full", "scan-small", "retrieve-small", "topk-small", "prefill-small",
@@ -77,6 +79,18 @@ def scan_bytes_per_launch(T, n_chunks, D, N, in_bytes=2, state_bytes=2):
     """Algorithmic HBM bytes of one encode launch: every input element read once
     (x, dt: T*D each; B: T*N), the captured state written once, the offsets and A read."""
     return T * (2 * D + N) * in_bytes + n_chunks * D * N * state_bytes + 8 * (n_chunks + 1) + 4 * D * N
+
+
+def host_available_bytes() -> int:
+    """MemAvailable of the host (0 if it cannot be read)."""
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    return int(line.split()[1]) * 1024
+    except OSError:
+        pass
+    return 0
 
 
 def peaks():
@@ -95,6 +109,10 @@ def peaks():
 # multiplies) and the 16 accumulations G_n += w_n * B_n (16 FMAs). The exponential E = 2^L
 # runs on the SFU and is not counted.
 ALU_OPS_PER_CHANNEL_TOKEN = 34
+# The direct update with a readout (y mode): the exponent argument dt * A[d,0] (1), u = dt * x
+# (1), the decay powers alpha_n = r^(n+1) (r^2 and 7 packed multiplies: 15), u * B_n (16),
+# h_n = alpha_n h_n + u B_n (16 FMAs) and y = sum_n C_n h_n (16 FMAs and one add: 17).
+ALU_OPS_DIRECT_Y = 66
 FP32_LANES_PER_SM = 128      # 4 sub-partitions x 32 FP32 lanes (FFMA and FFMA2 alike)
 FALLBACK_SM_MHZ = 2070.0
 
@@ -210,17 +228,18 @@ def whole_job_rate(units_per_rank_step: float, world: int, steps: int, seconds: 
 
 
 def run_reference(args):
-    """The oracle (fp64, sequential, one host core) on a bounded sample of the encode."""
+    """The oracle (fp64; each chunk a sequential rollout, chunks split over every host
+    core) on a bounded sample of the paper-shaped encode."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
-    import numpy as np
     import torch
 
     import oracle
     import synth
     shape = synth.PAPER
-    chunks, T = 1, shape.chunk_len
+    cores = os.cpu_count() or 1
+    chunks, T = 4 * cores, shape.chunk_len
     x, dt, A, B, _ = synth.host_scan_inputs(chunks * T, shape.D, shape.N, seed=0)
     # bf16 inputs, widened exactly, as the GPU path sees them
     bf = lambda a: torch.from_numpy(a).to(torch.bfloat16).double().numpy()
@@ -228,23 +247,23 @@ def run_reference(args):
     off = synth.fixed_offsets(chunks, T)
     oracle.build()
     for _ in range(args.warmup):
-        oracle.scan(x, dt, A, B, off)
+        oracle.scan_threads(x, dt, A, B, off, cores)
     times = []
     for _ in range(args.steps):
         t0 = time.perf_counter()
-        oracle.scan(x, dt, A, B, off)
+        oracle.scan_threads(x, dt, A, B, off, cores)
         times.append(time.perf_counter() - t0)
     per_layer = chunks * T / statistics.mean(times)
     value = per_layer / shape.n_layers          # tokens through all 24 layers per second
-    sample = (f"{chunks} chunk x {T} tokens x 1 layer of the paper-shaped encode (D=256, N=16), "
-              f"bf16-valued inputs in fp64; rate divided by 24 layers")
+    sample = (f"{chunks} chunks x {T} tokens x 1 layer of the paper-shaped encode (D=256, N=16) on "
+              f"{cores} host threads, bf16-valued inputs in fp64; rate divided by 24 layers")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * statistics.mean(times), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": "paper-shaped corpus encode (sampled for the CPU oracle)",
                        "chunk_tokens": T, "layers": shape.n_layers, "D": shape.D, "N": shape.N},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -508,6 +527,125 @@ def measure_extensions(pg, synth, torch, dev, layer_in, off, T, n_chunks, index,
     return out
 
 
+def measure_configs(pg, synth, torch, dev, hbm, alu_peak, cpu_chunks):
+    """The two other encode workloads, each on its own resident inputs (every launch
+    streams them from HBM; they are far above L2): the single-layer wide encode (D=2048,
+    1024 x 512 tokens; fp32 state capture, and a readout mode writing bf16 y) and one layer
+    of the ragged large-scale encode (D=512, 8192 chunks of U[256, 4096] tokens, bf16
+    bank; 24 such layers make the workload). Returns the rows and, for the CPU baseline,
+    the first ``cpu_chunks`` chunks of each workload's inputs copied back to the host."""
+    out, samples = {}, {}
+
+    def timed(fn, iters=5):
+        fn()
+        ts = []
+        for _ in range(iters):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            b.record()
+            b.synchronize()
+            ts.append(a.elapsed_time(b))
+        ts.sort()
+        return ts[len(ts) // 2]
+
+    for shape in (synth.WIDE, synth.RAGGED):
+        off_np = synth.shape_offsets(shape, 0)
+        T = int(off_np[-1])
+        inp = synth.device_scan_inputs(T, shape.D, shape.N, 0, 0, dev, with_C=shape is synth.WIDE)
+        off = torch.from_numpy(off_np).to(dev)
+        sdt = torch.float32 if shape is synth.WIDE else torch.bfloat16
+        states = torch.empty((shape.n_chunks, 1, shape.D, shape.N), dtype=sdt, device=dev)
+        si = pg.scan_inputs(inp["x"], inp["dt"], inp["B"], inp["A"], a_kind=pg.PRECOG_A_POWER)
+        ms = timed(lambda: pg.precog_encode_chunks(si, off, T, states_out=states))
+        nb = scan_bytes_per_launch(T, shape.n_chunks, shape.D, shape.N, state_bytes=states.element_size())
+        ct = T * shape.D
+        row = {"ms_per_layer": ms, "tokens": T, "chunks": shape.n_chunks, "D": shape.D,
+               "algorithmic_bytes": nb, "achieved_gbs": nb / (ms * 1e-3) / 1e9,
+               "frac_hbm": nb / (ms * 1e-3) / 1e9 / hbm,
+               "frac_alu": ALU_OPS_PER_CHANNEL_TOKEN * ct / (ms * 1e-3) / 1e12 / alu_peak,
+               "state_dtype": str(sdt).replace("torch.", "")}
+        if shape is synth.WIDE:
+            row["tokens_per_s"] = T / (ms * 1e-3)
+            out["wide_encode_capture"] = row
+            y = torch.empty((1, T, shape.D), dtype=torch.bfloat16, device=dev)
+            sy = pg.scan_inputs(inp["x"], inp["dt"], inp["B"], inp["A"], inp["C"], a_kind=pg.PRECOG_A_POWER)
+            ms = timed(lambda: pg.precog_encode_chunks(sy, off, T, states_out=states, y_out=y))
+            nb_y = nb + T * shape.N * 2 + T * shape.D * 2
+            out["wide_encode_y"] = {"ms_per_layer": ms, "tokens": T, "tokens_per_s": T / (ms * 1e-3),
+                                    "algorithmic_bytes": nb_y, "achieved_gbs": nb_y / (ms * 1e-3) / 1e9,
+                                    "frac_hbm": nb_y / (ms * 1e-3) / 1e9 / hbm,
+                                    "frac_alu": ALU_OPS_DIRECT_Y * ct / (ms * 1e-3) / 1e12 / alu_peak,
+                                    "alu_ops_per_channel_token": ALU_OPS_DIRECT_Y}
+            del y
+        else:
+            row["layers"] = shape.n_layers
+            row["tokens_per_s"] = T / (shape.n_layers * ms * 1e-3)   # through all 24 layers
+            out["ragged_encode"] = row
+        r1 = int(off_np[cpu_chunks])
+        samples[shape.name] = {k: inp[k][:r1].cpu().double().numpy() for k in ("x", "dt", "B")}
+        samples[shape.name]["A"] = inp["A"].cpu().double().numpy()
+        samples[shape.name]["offsets"] = off_np[:cpu_chunks + 1].copy()
+        samples[shape.name]["per_layer_tokens"] = T
+        samples[shape.name]["layers"] = shape.n_layers
+        del inp, states, si
+        torch.cuda.empty_cache()
+    return out, samples
+
+
+def cpu_baseline(oracle, paper, others, query, L):
+    """The oracle (fp64, sequential per chunk) on bounded samples of each workload, on
+    one host core and on every host core (chunks split over threads, each chunk the same
+    sequential rollout). Rates are extrapolated linearly: chunks and layers are
+    independent (Sec. 4.2)."""
+    oracle.build()
+    cores = os.cpu_count() or 1
+
+    def rate(sample, threads, chunks):
+        off = sample["offsets"][:chunks + 1]
+        r1 = int(off[-1])
+        args = (sample["x"][:r1], sample["dt"][:r1], sample["A"], sample["B"][:r1], off)
+        t0 = time.perf_counter()
+        if threads == 1:
+            oracle.scan(*args)
+        else:
+            oracle.scan_threads(*args, threads)
+        dt_s = time.perf_counter() - t0
+        return r1 / dt_s / sample["layers"], dt_s, r1
+
+    res = {"kind": "oracle", "unit": UNIT, "cores": cores}
+    one, s1, tok1 = rate(paper, 1, 16)
+    n_all = min(paper["offsets"].shape[0] - 1, 4 * cores)
+    allc, sa, toka = rate(paper, cores, n_all)
+    res.update(value=allc, seconds=sa,
+               sample=f"{n_all} chunks x 3000 tokens x 1 layer of the paper-shaped encode on {cores} host "
+                      f"threads (chunks split across threads, fp64 sequential rollout per chunk); rate "
+                      f"divided by {L} layers",
+               single_core={"value": one, "seconds": s1, "sample": "16 chunks x 3000 tokens x 1 layer, one core"})
+    for name, smp in others.items():
+        n = smp["offsets"].shape[0] - 1
+        o1, t1, _ = rate(smp, 1, n)
+        oa, ta, _ = rate(smp, cores, n)
+        res[name] = {"single_core": o1, "all_cores": oa, "seconds": [t1, ta],
+                     "sample": f"{n} chunks x 1 layer, rate divided by {smp['layers']} layer(s)"}
+    if query is not None:
+        t0 = time.perf_counter()
+        idx, _ = oracle.retrieve(query["index"], query["q"])
+        t_r = time.perf_counter() - t0
+        row = int(idx[0])
+        t0 = time.perf_counter()
+        for l in range(L):
+            oracle.rollout(query["x"][l], query["dt"][l], query["A"][l], query["B"][l], query["C"][l],
+                           h0=query["bank"][l], want_y=True)
+        t_p = time.perf_counter() - t0
+        res["query_path_q1"] = {"retrieve_s": t_r, "prefill_s": t_p, "latency_us": 1e6 * (t_r + t_p),
+                                "retrieved_planted": row == query["row"],
+                                "sample": "one query: exact retrieval over the full 1M x 768 index and "
+                                          f"the {L}-layer prefill of 64 tokens from the injected state, "
+                                          "one core"}
+    return res
+
+
 # ------------------------------------------------------------------------------ our arm
 
 
@@ -642,22 +780,30 @@ def main():
     avg_scan_ms = statistics.mean(scan_ms)
     achieved = bpl / (avg_scan_ms * 1e-3) / 1e9
     layer_traffic = profiled_traffic()
-    # The scan is bound by the FP32 FMA pipe (ncu: FMA pipe 66 % busy, DRAM 36 %), so the
-    # roofline is the ALU one; the HBM fraction the metric names is carried beside it.
+    # The metric's roofline: algorithmic HBM bytes per launch over the launch's CUDA-event
+    # time, against the measured copy bandwidth. The kernel's binding resource is the FP32
+    # FMA pipe (ncu: FMA pipe busy, DRAM far from saturated), so the FMA-pipe roofline is
+    # carried beside it, with the HBM fraction that pipe allows at 100 % busy.
     alu_peak, sms, mhz = alu_peak_tops(dev)
     ops = S * T * D * ALU_OPS_PER_CHANNEL_TOKEN
     alu_achieved = ops / (avg_scan_ms * 1e-3) / 1e12
-    roofline = {"bound": "alu", "achieved": alu_achieved, "peak": alu_peak,
-                "unit": "Tops/s (FP32 FMA-pipe lane operations)", "frac": alu_achieved / alu_peak,
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+                "peak_source": peak_src,
                 "traffic": None if layer_traffic is None else S * layer_traffic,
-                "peak_derivation": f"{sms} SMs x {FP32_LANES_PER_SM} FP32 lanes x {mhz:.0f} MHz",
-                "ops_per_channel_token": ALU_OPS_PER_CHANNEL_TOKEN, "algorithmic_ops_per_launch": ops,
-                "hbm": {"achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
-                        "peak_source": peak_src,
-                        "alu_ceiling_frac": alu_peak * 1e12 / ALU_OPS_PER_CHANNEL_TOKEN
+                "traffic_source": ("dram__bytes_read.sum + dram__bytes_write.sum of the ncu capture "
+                                   "summarised in profiles/scan_encode_paper_shaped.md (taken on this "
+                                   "scan.cu, scaled by tokens to one launch)") if layer_traffic is not None
+                else "null: the committed ncu capture was taken on another scan.cu",
+                "limiter": "alu",
+                "alu": {"achieved": alu_achieved, "peak": alu_peak,
+                        "unit": "Tops/s (FP32 FMA-pipe lane operations)", "frac": alu_achieved / alu_peak,
+                        "peak_derivation": f"{sms} SMs x {FP32_LANES_PER_SM} FP32 lanes x {mhz:.0f} MHz",
+                        "ops_per_channel_token": ALU_OPS_PER_CHANNEL_TOKEN,
+                        "algorithmic_ops_per_launch": ops,
+                        "hbm_frac_at_alu_peak": alu_peak * 1e12 / ALU_OPS_PER_CHANNEL_TOKEN
                         * (bpl / (S * T * D)) / (hbm * 1e9)},
                 "layers_per_launch": S,
-                "kernel": "scan_kernel (encode, capture)",
+                "kernel": "scan_kernel (encode, rescaled capture)",
                 "algorithmic_bytes_per_launch": bpl, "avg_launch_ms": avg_scan_ms}
 
     # ---------------- end to end: host inputs -> device -> encode/query -> host results
@@ -665,10 +811,17 @@ def main():
     # latency and extension phases are not part of it)
     e2e = None
     if not args.no_e2e:
-        host = {k: torch.empty(sets[0][k].shape, dtype=sets[0][k].dtype, pin_memory=True)
-                for k in ("x", "dt", "B")}
-        for k in host:
-            host[k].copy_(sets[0][k])
+        # one pinned host copy per resident input set, so that layer l streams set l mod S's
+        # inputs from the host and the e2e bank equals the timed region's
+        # (when the host cannot pin that much, the sets share one host copy)
+        set_bytes = sum(sets[0][k].numel() * sets[0][k].element_size() for k in ("x", "dt", "B"))
+        HS = S if host_available_bytes() > 2 * S * set_bytes else 1
+        host = [{k: torch.empty(sets[s_][k].shape, dtype=sets[s_][k].dtype, pin_memory=True)
+                 for k in ("x", "dt", "B")} for s_ in range(HS)]
+        for s_ in range(HS):
+            for k in host[s_]:
+                host[s_][k].copy_(sets[s_][k])
+        host = [host[s_ % HS] for s_ in range(S)]
         hq = {k: torch.empty(qb[k].shape, dtype=qb[k].dtype, pin_memory=True)
               for k in ("q", "x", "dt", "B", "C")}
         for k in hq:
@@ -678,7 +831,7 @@ def main():
                     for k in ("idx", "score", "y", "h")}
         copy_stream = torch.cuda.Stream(device=dev)
         comp = torch.cuda.current_stream(dev)
-        h2d = sum(host[k].numel() * host[k].element_size() for k in host) * L
+        h2d = sum(host[l % S][k].numel() * host[l % S][k].element_size() for l in range(L) for k in host[0])
         h2d += sum(hq[k].numel() * hq[k].element_size() for k in hq)
         d2h = bank.numel() * bank.element_size()
         d2h += sum(out_host[k].numel() * out_host[k].element_size() for k in out_host)
@@ -692,7 +845,7 @@ def main():
                     if done[l % S] is not None:
                         copy_stream.wait_event(done[l % S])
                     for k in ("x", "dt", "B"):
-                        buf[k].copy_(host[k], non_blocking=True)
+                        buf[k].copy_(host[l % S][k], non_blocking=True)
                     e = torch.cuda.Event()
                     e.record(copy_stream)
                 comp.wait_event(e)
@@ -716,7 +869,9 @@ def main():
         torch.cuda.synchronize()
         e2e_s = max_over_ranks(time.perf_counter() - w0)
         barrier()
+        bank_matches = bool(torch.equal(bank_host, bank.cpu()))
         e2e = {"value": whole_job_rate(tokens_per_step, world, args.e2e_steps, e2e_s), "unit": UNIT,
+               "host_input_sets": HS, "bank_equals_timed_region": bank_matches,
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                "ms_per_step": 1e3 * e2e_s / args.e2e_steps, "steps": args.e2e_steps,
                # the host link is shared with the machine's other GPUs: this rate (and so
@@ -783,25 +938,42 @@ def main():
     if st != 0:
         raise RuntimeError(f"device status {st} bits {bits:#x} after the timed region")
 
-    # ---------------- CPU baseline: the oracle on a bounded sample (rank 0, N=1 only)
+    # ---------------- CPU samples: the device-generated inputs of a few chunks (and of one
+    # query) copied back, so the oracle sees exactly the values the GPU saw
+    want_cpu = not args.no_cpu and rank == 0 and world == 1
+    cpu_paper = cpu_query = None
+    n_cpu = 16
+    if want_cpu:
+        n_paper = max(n_cpu, 4 * (os.cpu_count() or 1))
+        r1 = n_paper * shape.chunk_len
+        cpu_paper = {k: sets[0][k][:r1].cpu().double().numpy() for k in ("x", "dt", "B")}
+        cpu_paper.update(A=sets[0]["A"].cpu().double().numpy(), offsets=synth.fixed_offsets(n_paper, shape.chunk_len),
+                         layers=L)
+        q1 = query_batch(1, seed + 11)
+        prow = int(q1["rows"][0])
+        cpu_query = {"index": index.cpu().double().numpy(), "q": q1["q"].cpu().double().numpy(),
+                     "row": prow, "bank": qbank[prow].cpu().double().numpy(),
+                     **{k: q1[k].cpu().double().numpy() for k in ("x", "dt", "B", "C", "A")}}
+        del q1
+
+    # ---------------- the other encode configurations, on their own resident inputs
+    configs = None
+    if not args.no_configs:
+        del x_all, dt_all, B_all, sets, call_in, scan_in, qbank, index, bank, qb
+        torch.cuda.empty_cache()
+        alu_peak_v = alu_peak_tops(dev)[0]
+        configs, cfg_samples = measure_configs(pg, synth, torch, dev, peaks()[0], alu_peak_v, n_cpu)
+        st, bits = pg.precog_device_status()
+        if st != 0:
+            raise RuntimeError(f"device status {st} bits {bits:#x} after the configuration runs")
+    else:
+        cfg_samples = {}
+
+    # ---------------- CPU baseline: the oracle on bounded samples (rank 0, N=1 only)
     cpu = None
-    if not args.no_cpu and rank == 0 and world == 1:
+    if want_cpu:
         import oracle
-        chunks = 2
-        xs = sets[0]["x"][: chunks * shape.chunk_len].double().cpu().numpy()
-        dts = sets[0]["dt"][: chunks * shape.chunk_len].double().cpu().numpy()
-        Bs = sets[0]["B"][: chunks * shape.chunk_len].double().cpu().numpy()
-        An = sets[0]["A"].cpu().numpy()
-        offs = synth.fixed_offsets(chunks, shape.chunk_len)
-        oracle.build()
-        c0 = time.perf_counter()
-        oracle.scan(xs, dts, An, Bs, offs)
-        c_s = time.perf_counter() - c0
-        cpu = {"value": chunks * shape.chunk_len / c_s / L, "unit": UNIT, "cores": 1,
-               "kind": "oracle",
-               "sample": f"{chunks} chunks x {shape.chunk_len} tokens x 1 layer of this workload "
-                         f"(fp64 sequential oracle, one core), rate divided by {L} layers",
-               "seconds": c_s}
+        cpu = cpu_baseline(oracle, cpu_paper, cfg_samples, cpu_query, L)
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
@@ -818,7 +990,7 @@ def main():
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks,
                 "gpu_launches": int(launches), "latency": latency,
                 "retrieved_planted": ok_rows, "input_gen_s_per_layer": gen_s_per_layer,
-                "extensions": extras}
+                "configs": configs, "extensions": extras}
         print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()

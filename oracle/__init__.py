@@ -13,6 +13,8 @@ module compiles it with gcc and marshals numpy arrays into it.
 * :func:`retrieve` -- exact top-1 dot-product retrieval (Sec. 4.2), lowest row
   on ties, NaN never wins.
 * :func:`rollout` -- one chunk convenience wrapper of :func:`scan`.
+* :func:`scan_threads` -- :func:`scan` with the chunks split over host threads
+  (chunks are independent, Sec. 4.2); the per-chunk arithmetic is :func:`scan`'s.
 * :func:`retrieve_topk` -- the k best rows per query by exact score (ties to the
   lower row), the top-k of Sec. 4.2 / Sec. 5.4.
 * :func:`compose` -- the softmax-weighted state composition of Sec. 4.4
@@ -128,6 +130,33 @@ def scan(x, dt, A, B, offsets, C=None, h0=None, want_y=False):
     if rc != 0:
         raise ValueError(f"oracle_scan rejected its arguments (rc={rc})")
     return states, y
+
+
+def scan_threads(x, dt, A, B, offsets, threads: int):
+    """:func:`scan` (capture only, zero initial state) with the chunks split into
+    ``threads`` contiguous groups, each scanned by its own host thread. The C rollout
+    releases the interpreter lock while it runs, so the groups run on separate cores.
+    The arithmetic is :func:`scan`'s: every chunk's result is bit-identical to it.
+    Returns the ``[n_chunks, D, N]`` states."""
+    import concurrent.futures as cf
+    offsets = np.asarray(offsets, dtype=np.int64)
+    n_chunks = offsets.shape[0] - 1
+    x, dt, A, B = _f64(x), _f64(dt), _f64(A), _f64(B)
+    D, N = A.shape
+    states = np.zeros((n_chunks, D, N), dtype=np.float64)
+    bounds = np.linspace(0, n_chunks, max(1, min(threads, n_chunks)) + 1).astype(np.int64)
+
+    def part(i):
+        c0, c1 = int(bounds[i]), int(bounds[i + 1])
+        if c1 == c0:
+            return
+        r0, r1 = int(offsets[c0]), int(offsets[c1])
+        st, _ = scan(x[r0:r1], dt[r0:r1], A, B[r0:r1], offsets[c0:c1 + 1] - r0)
+        states[c0:c1] = st
+
+    with cf.ThreadPoolExecutor(max_workers=len(bounds) - 1) as ex:
+        list(ex.map(part, range(len(bounds) - 1)))
+    return states
 
 
 def rollout(x, dt, A, B, C=None, h0=None, want_y=False):

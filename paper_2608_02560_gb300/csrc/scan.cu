@@ -64,9 +64,13 @@ __device__ uint32_t g_scan_status;
 #ifndef PRECOG_FIXDS
 #define PRECOG_FIXDS 1
 #endif
-#ifndef PRECOG_E2_SFU
-#define PRECOG_E2_SFU 0
+#ifndef PRECOG_MIXED_U
+#define PRECOG_MIXED_U 1
 #endif
+#ifndef PRECOG_EARLY_EX2
+#define PRECOG_EARLY_EX2 1
+#endif
+
 
 constexpr int kN = 16;          // state size (N) supported by the kernels
 constexpr int kMaxSlice = 256;  // channels per CTA at most (the default slice)
@@ -360,17 +364,25 @@ __device__ __forceinline__ void renormalise(f2 (&g)[8], float &L) {
     L = 0.f;
 }
 
+// G_n += u * E^(n+1) * B_n
+__device__ __forceinline__ void accumulate_e(f2 (&g)[8], const f2 (&b)[8], float u, float E) {
+    const float w0 = u * E;
+    const float E2 = E * E;
+    f2 w = pack2(w0, w0 * E);
+    const f2 ee = pack2(E2, E2);
+    g[0] = fma2(w, b[0], g[0]);
+#pragma unroll
+    for (int i = 1; i < 8; ++i) {
+        w = mul2(w, ee);
+        g[i] = fma2(w, b[i], g[i]);
+    }
+}
+
 // G_n += u * 2^((n+1) * Ln) * B_n
 __device__ __forceinline__ void accumulate(f2 (&g)[8], const f2 (&b)[8], float u, float Ln) {
     const float E = ex2(Ln);
     const float w0 = u * E;
-#if PRECOG_E2_SFU
-    // 2^(2 Ln) from the SFU: doubling Ln exactly by an exponent-field add (|Ln| <= kLmax
-    // here, or 0; a zero becomes 2^-126, whose exponential is 1 as well)
-    const float E2 = ex2(__int_as_float(__float_as_int(Ln) + 0x00800000));
-#else
     const float E2 = E * E;
-#endif
     f2 w = pack2(w0, w0 * E);
     const f2 ee = pack2(E2, E2);
     g[0] = fma2(w, b[0], g[0]);
@@ -453,48 +465,94 @@ __device__ __forceinline__ void renorm_floor(f2 (&g)[8], float &L) {
 // whole window goes through the per-token check.
 constexpr int kGroup = PRECOG_RESCALED_GROUP;
 
+// dt * x of the low (high) bf16 halves of two words, exact in fp32 (a product of two
+// 8-bit significands), by the mixed-precision FMA with -0 as addend: no widening.
+__device__ __forceinline__ float mul_bf16_lo(uint32_t a, uint32_t b) {
+    float d;
+    asm("{ .reg .b16 al, ah, bl, bh; mov.b32 {al, ah}, %1; mov.b32 {bl, bh}, %2;"
+        " fma.rn.f32.bf16 %0, al, bl, %3; }"
+        : "=f"(d) : "r"(a), "r"(b), "f"(-0.0f));
+    return d;
+}
+__device__ __forceinline__ float mul_bf16_hi(uint32_t a, uint32_t b) {
+    float d;
+    asm("{ .reg .b16 al, ah, bl, bh; mov.b32 {al, ah}, %1; mov.b32 {bl, bh}, %2;"
+        " fma.rn.f32.bf16 %0, ah, bh, %3; }"
+        : "=f"(d) : "r"(a), "r"(b), "f"(-0.0f));
+    return d;
+}
+
+template <int CPT>
+__device__ __forceinline__ void load_words(const unsigned char *p, uint32_t (&w)[CPT / 2]) {
+    if constexpr (CPT == 2) {
+        w[0] = *reinterpret_cast<const uint32_t *>(p);
+    } else {
+        const uint2 q = *reinterpret_cast<const uint2 *>(p);
+        w[0] = q.x;
+        w[1] = q.y;
+    }
+}
+
+template <int CPT>
+__device__ __forceinline__ void widen_words(const uint32_t (&w)[CPT / 2], float (&v)[CPT]) {
+#pragma unroll
+    for (int i = 0; i < CPT / 2; ++i) {
+        v[2 * i] = __uint_as_float(w[i] << 16);
+        v[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+    }
+}
+
 template <class C>
 __device__ __forceinline__ void scan_tile_rescaled(const unsigned char *st, const StageLayout &lay,
-                                                   int DS, int dl, int t0, int ntok,
+                                                   const float *bsrc, int DS, int dl, int t0, int ntok,
                                                    f2 (&g)[C::CPT][8], float (&L)[C::CPT],
                                                    const float (&kk)[C::CPT], unsigned wmask) {
     constexpr int CPT = C::CPT;
     using TIn = typename C::TIn;
-    const float *bsrc = reinterpret_cast<const float *>(st + (C::CONV ? lay.bf : lay.bs));
+    // 16-bit inputs: dt is kept as raw words across the vote, and u = dt * x is formed
+    // from the raw halves
+    constexpr bool MIX = PRECOG_MIXED_U && C::CONV;
     int t = t0;
     for (; t + kGroup <= ntok; t += kGroup) {
         float dvk[kGroup][CPT], Lk[kGroup][CPT];
+        uint32_t dw[kGroup][CPT / 2];
         uint32_t neg = 0;
 #pragma unroll
         for (int k = 0; k < kGroup; ++k) {
-            uint32_t nk;
-            load_chan<TIn, CPT>(st + lay.dts + ((t + k) * DS + dl) * C::SZ, dvk[k], nk);
-            neg |= nk;
+            if constexpr (MIX) {
+                load_words<CPT>(st + lay.dts + ((t + k) * DS + dl) * C::SZ, dw[k]);
+                widen_words<CPT>(dw[k], dvk[k]);
+#pragma unroll
+                for (int i = 0; i < CPT / 2; ++i) neg |= dw[k][i];
+            } else {
+                uint32_t nk;
+                load_chan<TIn, CPT>(st + lay.dts + ((t + k) * DS + dl) * C::SZ, dvk[k], nk);
+                neg |= nk;
+            }
 #pragma unroll
             for (int j = 0; j < CPT; ++j) Lk[k][j] = fmaf(dvk[k][j], kk[j], k ? Lk[k - 1][j] : L[j]);
         }
+        if constexpr (MIX) neg &= 0x80008000u;
         bool up = false;
 #pragma unroll
         for (int j = 0; j < CPT; ++j) up |= !(Lk[kGroup - 1][j] <= kLmax);
         bool slow = false;
         if (__any_sync(wmask, up || neg != 0)) {
-#if PRECOG_RENORM_FLOOR
             slow = __any_sync(wmask, neg != 0);
             if (!slow) {
 #pragma unroll
                 for (int j = 0; j < CPT; ++j) renorm_floor(g[j], L[j]);
                 bool up2 = false;
 #pragma unroll
-                for (int k = 0; k < kGroup; ++k)
+                for (int k = 0; k < kGroup; ++k) {
+                    if constexpr (MIX) widen_words<CPT>(dw[k], dvk[k]);
 #pragma unroll
                     for (int j = 0; j < CPT; ++j) Lk[k][j] = fmaf(dvk[k][j], kk[j], k ? Lk[k - 1][j] : L[j]);
+                }
 #pragma unroll
                 for (int j = 0; j < CPT; ++j) up2 |= !(Lk[kGroup - 1][j] <= kLmax);
                 slow = __any_sync(wmask, up2);
             }
-#else
-            slow = true;
-#endif
         }
         if (slow) {
             // unrolled so that dvk stays in registers (no dynamic indexing)
@@ -505,18 +563,45 @@ __device__ __forceinline__ void scan_tile_rescaled(const unsigned char *st, cons
                 uint32_t nx;
                 load_b(bsrc, t + k, b);
                 load_chan<TIn, CPT>(st + lay.xs + ((t + k) * DS + dl) * C::SZ, xv, nx);
+                if constexpr (MIX) widen_words<CPT>(dw[k], dvk[k]);
                 token_checked<CPT>(g, L, kk, b, xv, dvk[k], wmask);
             }
         } else {
+#if PRECOG_EARLY_EX2
+            float Ek[kGroup][CPT];
+#pragma unroll
+            for (int k = 0; k < kGroup; ++k)
+#pragma unroll
+                for (int j = 0; j < CPT; ++j) Ek[k][j] = ex2(Lk[k][j]);
+#endif
 #pragma unroll
             for (int k = 0; k < kGroup; ++k) {
                 f2 b[8];
-                float xv[CPT];
-                uint32_t nx;
                 load_b(bsrc, t + k, b);
-                load_chan<TIn, CPT>(st + lay.xs + ((t + k) * DS + dl) * C::SZ, xv, nx);
+                float u[CPT];
+                if constexpr (MIX) {
+                    uint32_t xw[CPT / 2];
+                    load_words<CPT>(st + lay.xs + ((t + k) * DS + dl) * C::SZ, xw);
 #pragma unroll
-                for (int j = 0; j < CPT; ++j) accumulate(g[j], b, dvk[k][j] * xv[j], Lk[k][j]);
+                    for (int i = 0; i < CPT / 2; ++i) {
+                        u[2 * i] = mul_bf16_lo(dw[k][i], xw[i]);
+                        u[2 * i + 1] = mul_bf16_hi(dw[k][i], xw[i]);
+                    }
+                } else {
+                    float xv[CPT];
+                    uint32_t nx;
+                    load_chan<TIn, CPT>(st + lay.xs + ((t + k) * DS + dl) * C::SZ, xv, nx);
+#pragma unroll
+                    for (int j = 0; j < CPT; ++j) u[j] = dvk[k][j] * xv[j];
+                }
+#pragma unroll
+                for (int j = 0; j < CPT; ++j) {
+#if PRECOG_EARLY_EX2
+                    accumulate_e(g[j], b, u[j], Ek[k][j]);
+#else
+                    accumulate(g[j], b, u[j], Lk[k][j]);
+#endif
+                }
             }
 #pragma unroll
             for (int j = 0; j < CPT; ++j) L[j] = Lk[kGroup - 1][j];
@@ -760,7 +845,8 @@ __global__ void __launch_bounds__(C::LB_THREADS, C::LB_BLOCKS)
             int t = 0;
             while (t < ntok) {
                 const int seg = static_cast<int>(min64(ntok - t, tcur.left));
-                scan_tile_rescaled<C>(st, lay, DS, dl, t, t + seg, h, Lw, kk, wmask);
+                scan_tile_rescaled<C>(st, lay, reinterpret_cast<const float *>(st + (C::CONV ? lay.bf : lay.bs)), DS, dl, t,
+                                      t + seg, h, Lw, kk, wmask);
                 t += seg;
                 tcur.left -= seg;
                 if (tcur.left == 0 || k * TILE + t == len) {
@@ -777,7 +863,8 @@ __global__ void __launch_bounds__(C::LB_THREADS, C::LB_BLOCKS)
                 }
             }
         } else if constexpr (C::RESCALED) {
-            scan_tile_rescaled<C>(st, lay, DS, dl, 0, ntok, h, Lw, kk, wmask);
+            scan_tile_rescaled<C>(st, lay, reinterpret_cast<const float *>(st + (C::CONV ? lay.bf : lay.bs)), DS, dl, 0,
+                                  ntok, h, Lw, kk, wmask);
         } else {
             scan_tile_direct<C>(st, lay, DS, dl, ntok, h, kpow, kgen, yrow, p.y_dtype, y_stride, p, tcur,
                                 len - k * TILE, p.layer0 + layer, d0 + dl);
@@ -861,10 +948,11 @@ cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
         // the corpus encode of 256-channel rows (the paper's layer width) gets a slice fixed
         // at compile time
         if constexpr (!HAS_H0 && !std::is_same<TIn, float>::value)
-            if (pick_slice(p.D, sizeof(TIn), PRECOG_RESCALED_CPT, kWideSlice) == 256)
-                return launch_cfg<Cfg<TIn, false, false, MODE, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
-                                      PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB, kTrajNone, kWideSlice,
-                                      256>>(p, stream);
+            if (pick_slice(p.D, sizeof(TIn), PRECOG_RESCALED_CPT, kWideSlice) == 256) {
+                using C256 = Cfg<TIn, false, false, MODE, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
+                                 PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB, kTrajNone, kWideSlice, 256>;
+                return launch_cfg<C256>(p, stream);
+            }
 #endif
         return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
                               PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB, kTrajNone, kWideSlice>>(p, stream);

@@ -457,3 +457,13 @@ def test_complex_scan_theorem1_and_geometric_series():
     a = np.exp(delta * (A_re + 1j * A_im))
     beta = (delta * xi)[:, None] * b[None, :]
     np.testing.assert_allclose(hs[0], a ** T * h0[0] + beta * (1 - a ** T) / (1 - a), rtol=1e-12)
+
+
+def test_scan_threads_matches_scan_bit_for_bit():
+    """The threaded driver only splits chunks over host threads: ragged and empty chunks
+    give exactly scan's states, for any thread count."""
+    x, dt, A, B, _ = synth.host_scan_inputs(1300, 32, 16, seed=5)
+    off = np.array([0, 300, 300, 650, 651, 1200, 1300], dtype=np.int64)
+    ref, _ = oracle.scan(x, dt, A, B, off)
+    for threads in (1, 2, 4, 9):
+        assert np.array_equal(oracle.scan_threads(x, dt, A, B, off, threads), ref)
