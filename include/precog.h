@@ -42,8 +42,13 @@ typedef enum precog_status {
     PRECOG_ERR_UNSUPPORTED = 2,  /* valid, but outside what the kernels implement */
     PRECOG_ERR_CUDA = 3,         /* a CUDA runtime call or a launch failed */
     PRECOG_ERR_TIMEOUT = 4,      /* a bounded device-side wait gave up */
-    PRECOG_ERR_DEVICE = 5        /* the device flagged bad offsets or bank rows */
+    PRECOG_ERR_DEVICE = 5        /* the device flagged bad offsets, bank rows, slots or A */
 } precog_status;
+/* Status 5 reports what only the device can see (precog_device_status: bad offsets, a
+ * bank row or slot outside its table, a false PRECOG_A_POWER statement). A retrieval
+ * with no comparable score (an empty index, or every score NaN) is not an error: it
+ * returns PRECOG_OK with row -1 and score NaN, a well-defined "no context" result that
+ * injects the zero state. There is no separate numeric-failure status. */
 
 typedef enum precog_dtype {
     PRECOG_F32 = 0,
@@ -169,7 +174,8 @@ precog_status precog_encode_trajectory(const precog_scan_inputs *in, const int64
  * (unit-norm keys and queries make this the cosine similarity of the paper).
  * Exact top-1, not an approximate index. Scores accumulate in fp32 from the
  * stored values; ties go to the lowest row; a NaN score never wins; if no row
- * has a comparable score the result is index -1 and score NaN.
+ * has a comparable score (M == 0, or every score NaN) the result is index -1 and
+ * score NaN, and the call still returns PRECOG_OK.
  *
  *   index          device [M][dim] keys in index_dtype (F16, BF16 or F32)
  *   queries        device [n_queries][dim], same dtype as the index
@@ -198,9 +204,10 @@ size_t precog_retrieve_workspace_size(int64_t M, int32_t dim, int32_t n_queries)
  * without the workspace: the partial keys go to a fixed 2 MiB array compiled
  * into the library, which every GPU that loads the library holds until exit.
  *   - Allocates nothing and calls no allocating routine.
- *   - The first call on a device looks up that array's device address (once
- *     per device, with the device current); make that first call before any
- *     stream capture.
+ *   - The first call in a CUDA context looks up that array's device address in
+ *     that context (once per context, with the context current; a reset device
+ *     or another context of the same device gets its own lookup); make that
+ *     first call before any stream capture.
  *   - Calls whose sizes need more than the 2 MiB (keys = precog_retrieve
  *     workspace bytes / 8; about 430 queries per call at any M on a 152-SM GPU)
  *     return PRECOG_ERR_UNSUPPORTED without launching anything.

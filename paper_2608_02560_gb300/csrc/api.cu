@@ -563,25 +563,68 @@ namespace {
 constexpr size_t kNoallocKeys = 262144;
 static __device__ __align__(256) unsigned long long g_noalloc_scratch[kNoallocKeys];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_noalloc_mutex;
-void *g_noalloc_ptr[kMaxDevices] = {};
+// The array's device address belongs to one CUDA context: after cudaDeviceReset, or
+// when a caller makes another context of the same device current, it is another
+// address. So the address is looked up once per context (keyed by the driver's unique
+// context id), not once per device number.
+using CtxGetCurrentFn = CUresult (*)(CUcontext *);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long *);
 
-// Device address of the scratch on the current device (set up once per device).
+template <typename F>
+F driver_fn(const char *name) {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion(name, &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+        return reinterpret_cast<F>(p);
+    return nullptr;
+}
+
+// Unique id of the calling thread's current context; false if there is none yet or the
+// driver cannot tell.
+bool current_context_id(unsigned long long *id) {
+    static const CtxGetCurrentFn get_current = driver_fn<CtxGetCurrentFn>("cuCtxGetCurrent");
+    static const CtxGetIdFn get_id = driver_fn<CtxGetIdFn>("cuCtxGetId");
+    if (get_current == nullptr || get_id == nullptr) return false;
+    CUcontext ctx = nullptr;
+    if (get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr) return false;
+    return get_id(ctx, id) == CUDA_SUCCESS;
+}
+
+struct NoallocSlot {
+    unsigned long long ctx_id;
+    void *ptr;
+};
+constexpr int kNoallocSlots = 64;
+std::mutex g_noalloc_mutex;
+NoallocSlot g_noalloc_slots[kNoallocSlots];
+int g_noalloc_filled = 0, g_noalloc_next = 0;
+
+// Device address of the scratch in the current context. The first call in a context
+// asks the runtime (cudaGetSymbolAddress, a host-side lookup that allocates nothing);
+// later calls in that context reuse the answer. Without context ids every call asks.
 precog_status noalloc_scratch(void **ptr) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
-    if (dev < 0 || dev >= kMaxDevices)
-        return fail(PRECOG_ERR_UNSUPPORTED, "device ordinal %d is beyond %d", dev, kMaxDevices);
-    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
-    if (g_noalloc_ptr[dev] == nullptr) {
-        void *p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-        if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(scratch)");
-        g_noalloc_ptr[dev] = p;
+    unsigned long long id = 0;
+    bool have_id = current_context_id(&id);
+    if (have_id) {
+        std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+        for (int i = 0; i < g_noalloc_filled; ++i)
+            if (g_noalloc_slots[i].ctx_id == id) {
+                *ptr = g_noalloc_slots[i].ptr;
+                return PRECOG_OK;
+            }
     }
-    *ptr = g_noalloc_ptr[dev];
+    void *p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(scratch)");
+    if (!have_id) have_id = current_context_id(&id);   // the lookup may have created the context
+    if (have_id) {
+        std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+        g_noalloc_slots[g_noalloc_next] = NoallocSlot{id, p};
+        g_noalloc_next = (g_noalloc_next + 1) % kNoallocSlots;
+        if (g_noalloc_filled < kNoallocSlots) ++g_noalloc_filled;
+    }
+    *ptr = p;
     return PRECOG_OK;
 }
 

@@ -39,33 +39,17 @@ __device__ __forceinline__ unsigned long long make_key(float s, int64_t row) {
            static_cast<unsigned long long>(0xffffffffu - static_cast<uint32_t>(row));
 }
 
+// The CUDA-core kernels take fp32 keys (16-bit keys go to the tensor cores).
 template <typename T> struct Vec;
-template <> struct Vec<__half> { static constexpr int n = 8; };
-template <> struct Vec<__nv_bfloat16> { static constexpr int n = 8; };
 template <> struct Vec<float> { static constexpr int n = 4; };
 
 template <typename T>
 __device__ __forceinline__ void widen(const uint4 &v, float (&f)[Vec<T>::n]) {
-    if constexpr (std::is_same<T, float>::value) {
-        f[0] = __uint_as_float(v.x);
-        f[1] = __uint_as_float(v.y);
-        f[2] = __uint_as_float(v.z);
-        f[3] = __uint_as_float(v.w);
-    } else {
-        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            if constexpr (std::is_same<T, __half>::value) {
-                const __half2 h2 = *reinterpret_cast<const __half2 *>(&w[i]);
-                const float2 f2v = __half22float2(h2);
-                f[2 * i] = f2v.x;
-                f[2 * i + 1] = f2v.y;
-            } else {
-                f[2 * i] = __uint_as_float(w[i] << 16);
-                f[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
-            }
-        }
-    }
+    static_assert(std::is_same<T, float>::value, "fp32 keys only");
+    f[0] = __uint_as_float(v.x);
+    f[1] = __uint_as_float(v.y);
+    f[2] = __uint_as_float(v.z);
+    f[3] = __uint_as_float(v.w);
 }
 
 // partial[blockIdx.x * n_queries + q] = best key of this CTA for query q.
@@ -393,16 +377,12 @@ cudaError_t launch_gemv(const RetrieveParams &p, cudaStream_t stream, int grid, 
     return e;
 }
 
-// Batches larger than one GEMV pass run on the tensor cores (16-bit keys).
 // 16-bit indexes go to the tensor cores: one pass over the keys for up to 256 queries,
 // streamed by TMA; even a single query's pass is a little faster there (0.246 vs 0.266
-// ms over 1M x 768 fp16 keys) than on the CUDA-core kernel, which needs a pass per 4
-// queries. fp32 indexes stay on the CUDA cores.
-constexpr int kTcMinQueries = 1;
-
-bool use_tc(const RetrieveParams &p) {
-    return p.dtype != PRECOG_F32 && p.n_queries >= kTcMinQueries && p.M > 0;
-}
+// ms over 1M x 768 fp16 keys) than a CUDA-core GEMV, which needs a pass per 4 queries.
+// fp32 indexes stay on the CUDA cores (the GEMV kernels below are instantiated for fp32
+// keys only).
+bool use_tc(const RetrieveParams &p) { return p.dtype != PRECOG_F32; }
 
 template <typename T, int VPL>
 cudaError_t launch_topk_pass(const RetrieveParams &p, int grid, int q, cudaStream_t stream) {
@@ -442,18 +422,14 @@ cudaError_t launch_retrieve(const RetrieveParams &p, cudaStream_t stream) {
     const int sz = p.dtype == PRECOG_F32 ? 4 : 2;
     if (p.dim * sz / 16 > kMaxVecsPerRow) return cudaErrorInvalidValue;
     uint64_t launches = 0;
-    cudaError_t e;
-    int parts;
-    if (use_tc(p)) {
+    cudaError_t e = cudaSuccess;
+    int parts = 0;  // an empty index has no partial keys: the finalize writes row -1, score NaN
+    if (p.M > 0 && use_tc(p)) {
         parts = retrieve_tc_grid(p.M, num_sms());
         e = launch_retrieve_tc(p, parts, stream, &launches);
-    } else {
+    } else if (p.M > 0) {
         parts = gemv_grid(p.M);
-        switch (p.dtype) {
-            case PRECOG_F16: e = launch_gemv<__half>(p, stream, parts, &launches); break;
-            case PRECOG_BF16: e = launch_gemv<__nv_bfloat16>(p, stream, parts, &launches); break;
-            default: e = launch_gemv<float>(p, stream, parts, &launches); break;
-        }
+        e = launch_gemv<float>(p, stream, parts, &launches);
     }
     if (e == cudaSuccess) {
         finalize_kernel<<<(p.n_queries + 3) / 4, 128, 0, stream>>>(
@@ -487,18 +463,14 @@ cudaError_t launch_retrieve_topk(const RetrieveParams &p, int k, cudaStream_t st
     const int sz = p.dtype == PRECOG_F32 ? 4 : 2;
     if (p.dim * sz / 16 > kMaxVecsPerRow || k < 1 || k > kListK) return cudaErrorInvalidValue;
     uint64_t launches = 0;
-    cudaError_t e;
-    int parts;
-    if (use_tc(p)) {
+    cudaError_t e = cudaSuccess;
+    int parts = 0;  // an empty index has no partial lists: the finalize writes rows -1
+    if (p.M > 0 && use_tc(p)) {
         parts = retrieve_tc_grid(p.M, num_sms());
         e = launch_retrieve_tc_topk(p, k, parts, stream, &launches);
-    } else {
+    } else if (p.M > 0) {
         parts = gemv_grid(p.M);
-        switch (p.dtype) {
-            case PRECOG_F16: e = launch_gemv_topk<__half>(p, stream, parts, &launches); break;
-            case PRECOG_BF16: e = launch_gemv_topk<__nv_bfloat16>(p, stream, parts, &launches); break;
-            default: e = launch_gemv_topk<float>(p, stream, parts, &launches); break;
-        }
+        e = launch_gemv_topk<float>(p, stream, parts, &launches);
     }
     if (e == cudaSuccess) {
         finalize_topk_kernel<<<(p.n_queries + 3) / 4, 128, 0, stream>>>(

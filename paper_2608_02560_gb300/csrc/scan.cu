@@ -58,18 +58,6 @@ __device__ uint32_t g_scan_status;
 #ifndef PRECOG_RESCALED_GROUP
 #define PRECOG_RESCALED_GROUP 4
 #endif
-#ifndef PRECOG_RENORM_FLOOR
-#define PRECOG_RENORM_FLOOR 1
-#endif
-#ifndef PRECOG_FIXDS
-#define PRECOG_FIXDS 1
-#endif
-#ifndef PRECOG_MIXED_U
-#define PRECOG_MIXED_U 1
-#endif
-#ifndef PRECOG_EARLY_EX2
-#define PRECOG_EARLY_EX2 1
-#endif
 
 
 constexpr int kN = 16;          // state size (N) supported by the kernels
@@ -511,7 +499,7 @@ __device__ __forceinline__ void scan_tile_rescaled(const unsigned char *st, cons
     using TIn = typename C::TIn;
     // 16-bit inputs: dt is kept as raw words across the vote, and u = dt * x is formed
     // from the raw halves
-    constexpr bool MIX = PRECOG_MIXED_U && C::CONV;
+    constexpr bool MIX = C::CONV;
     int t = t0;
     for (; t + kGroup <= ntok; t += kGroup) {
         float dvk[kGroup][CPT], Lk[kGroup][CPT];
@@ -567,13 +555,12 @@ __device__ __forceinline__ void scan_tile_rescaled(const unsigned char *st, cons
                 token_checked<CPT>(g, L, kk, b, xv, dvk[k], wmask);
             }
         } else {
-#if PRECOG_EARLY_EX2
+            // the group's exponentials first, so that their latency overlaps the rest
             float Ek[kGroup][CPT];
 #pragma unroll
             for (int k = 0; k < kGroup; ++k)
 #pragma unroll
                 for (int j = 0; j < CPT; ++j) Ek[k][j] = ex2(Lk[k][j]);
-#endif
 #pragma unroll
             for (int k = 0; k < kGroup; ++k) {
                 f2 b[8];
@@ -595,13 +582,7 @@ __device__ __forceinline__ void scan_tile_rescaled(const unsigned char *st, cons
                     for (int j = 0; j < CPT; ++j) u[j] = dvk[k][j] * xv[j];
                 }
 #pragma unroll
-                for (int j = 0; j < CPT; ++j) {
-#if PRECOG_EARLY_EX2
-                    accumulate_e(g[j], b, u[j], Ek[k][j]);
-#else
-                    accumulate(g[j], b, u[j], Lk[k][j]);
-#endif
-                }
+                for (int j = 0; j < CPT; ++j) accumulate_e(g[j], b, u[j], Ek[k][j]);
             }
 #pragma unroll
             for (int j = 0; j < CPT; ++j) L[j] = Lk[kGroup - 1][j];
@@ -944,7 +925,6 @@ cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
         else
             return launch_cfg<Cfg<TIn, false, false, MODE, 2, 16, 4, 3, kTrajDirect>>(p, stream);
     } else if constexpr (MODE == kPower && !HAS_Y) {
-#if PRECOG_FIXDS
         // the corpus encode of 256-channel rows (the paper's layer width) gets a slice fixed
         // at compile time
         if constexpr (!HAS_H0 && !std::is_same<TIn, float>::value)
@@ -953,7 +933,6 @@ cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
                                  PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB, kTrajNone, kWideSlice, 256>;
                 return launch_cfg<C256>(p, stream);
             }
-#endif
         return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
                               PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB, kTrajNone, kWideSlice>>(p, stream);
     } else {

@@ -62,7 +62,9 @@ def test_tiny_planted(cuda_device):
 @pytest.mark.parametrize("M,Q", [(1, 1), (5, 3), (1000, 9), (4099, 2)])
 def test_small_exact_integer_scores(cuda_device, dtype_name, M, Q):
     """Small-integer keys make every score exact in fp32: indices and scores must equal
-    the oracle's bit for bit, including the many exact ties (lowest row wins)."""
+    the oracle's bit for bit, including the many exact ties (lowest row wins). fp16 and
+    bf16 keys run the tensor-core kernel (every 16-bit retrieval does, a single query
+    included), fp32 keys the CUDA-core GEMV."""
     import torch
     dtype = getattr(torch, dtype_name)
     rng = np.random.default_rng(M * 7 + Q)
@@ -97,11 +99,16 @@ def test_ties_across_the_grid_and_nan_rows(cuda_device):
     assert list(idx) == [-1, -1] and np.all(np.isnan(score))
 
 
-def test_empty_index(cuda_device):
+@pytest.mark.parametrize("dtype_name", ["float16", "bfloat16", "float32"])
+def test_empty_index(cuda_device, dtype_name):
+    """An index without rows has no comparable score: row -1 and a NaN score for every
+    query (no sweep kernel runs; the merge alone writes the result)."""
     import torch
-    idx, score = _run(torch.empty((0, 64), dtype=torch.float16, device=cuda_device),
-                      torch.ones((3, 64), dtype=torch.float16, device=cuda_device))
+    dtype = getattr(torch, dtype_name)
+    idx, score = _run(torch.empty((0, 64), dtype=dtype, device=cuda_device),
+                      torch.ones((3, 64), dtype=dtype, device=cuda_device))
     assert list(idx) == [-1, -1, -1]
+    assert np.isnan(score).all()
 
 
 @pytest.mark.parametrize("Q", [1, 256])
@@ -126,7 +133,7 @@ def test_query_workload_full_index(cuda_device, Q):
     torch.cuda.empty_cache()
 
 
-# ------------------------------------------------------------- tensor-core path (16-bit keys, Q >= 2)
+# ------------------------------------------------------------- tensor-core path (every 16-bit retrieval)
 
 
 @pytest.mark.parametrize("dtype_name", ["float16", "bfloat16"])
@@ -134,8 +141,9 @@ def test_query_workload_full_index(cuda_device, Q):
                                      (4099, 300, 96), (20000, 17, 136), (3000, 2, 64), (70000, 4, 768),
                                      (513, 127, 64), (513, 128, 64)])
 def test_tensor_core_exact_integer_scores(cuda_device, dtype_name, M, Q, dim):
-    """Batches of five or more queries over a 16-bit index take the tcgen05 path. Small
-    integer keys and queries make every score exact in fp32, so indices and scores must
+    """Every retrieval over a 16-bit index takes the tcgen05 path; these shapes stress
+    its tiling. Small integer keys and queries make every score exact in fp32, so indices
+    and scores must
     equal the oracle's bit for bit: ragged tiles (M), ragged and multi-pass query batches
     (Q > 128, Q > 256), a K tail (dim not a multiple of 64), many exact ties."""
     import torch

@@ -5,6 +5,8 @@ workloads (single-layer wide encode, paper-shaped encode, ragged large-scale enc
 in the launch configuration the benchmark times, and sampled chunks are compared with
 the oracle one by one on inputs copied back from the device generator.
 """
+import os
+
 import numpy as np
 import pytest
 
@@ -277,38 +279,65 @@ def test_rescaled_renormalisation_regimes(cuda_device, scale, dt_shift):
 # ------------------------------------------------------------- full-size workloads, sampled
 
 
-def _sampled_check(dev, shape, layer, sample_chunks, y_mode=False, seed=0):
+def _sample(n_chunks, fixed, count=32, seed=0, last=64):
+    """The listed chunks, ``count`` seeded random ones, and four of the last ``last``
+    chunks (the launch's last wave)."""
+    rng = np.random.default_rng(1000 + seed)
+    pick = set(int(c) for c in fixed) | set(int(c) for c in rng.choice(n_chunks, count, replace=False))
+    pick |= set(int(c) for c in rng.choice(np.arange(n_chunks - last, n_chunks), 4, replace=False))
+    return sorted(pick)
+
+
+def _oracle_states(x, dt, B, A, off_np, chunks):
+    """Oracle final states of the listed chunks of one layer (inputs copied back from the
+    device exactly), the chunks split over host threads."""
+    import torch
+    rows = np.concatenate([np.arange(off_np[c], off_np[c + 1]) for c in chunks])
+    it = torch.from_numpy(rows).to(x.device)
+    lens = np.array([off_np[c + 1] - off_np[c] for c in chunks], dtype=np.int64)
+    sub_off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    return oracle.scan_threads(to_np(x[it]), to_np(dt[it]), A, to_np(B[it]), sub_off, os.cpu_count() or 1)
+
+
+def _sampled_check(dev, shape, layer, sample_chunks, y_mode=False, seed=0, state_dtype=None):
     """Generate one layer of a workload on the device at full size, run the encode as the
-    benchmark does, copy back the sampled chunks' inputs and compare with the oracle."""
+    benchmark does into a bank filled with NaN, check that exactly the layer's entries were
+    written (all finite) and compare the sampled chunks with the oracle. A bf16 bank is
+    held to the tolerance before its one rounding (half a bf16 ulp allowed), an fp32 one to
+    the plain tolerance."""
     import torch
     pg = _pg()
+    sdt = torch.bfloat16 if state_dtype is None else state_dtype
     off_np = synth.shape_offsets(shape, seed)
     T = int(off_np[-1])
     inp = synth.device_scan_inputs(T, shape.D, shape.N, seed, layer, dev, with_C=y_mode)
     off = torch.from_numpy(off_np).to(dev)
-    states = torch.empty((shape.n_chunks, shape.n_layers, shape.D, shape.N), dtype=torch.bfloat16,
-                         device=dev)
+    L_bank, slot = shape.n_layers, layer
+    states = torch.full((shape.n_chunks, L_bank, shape.D, shape.N), float("nan"), dtype=sdt, device=dev)
     y = torch.empty((1, T, shape.D), dtype=torch.bfloat16, device=dev) if y_mode else None
     pg.precog_encode_chunks(pg.scan_inputs(inp["x"], inp["dt"], inp["B"], inp["A"],
                                            inp.get("C") if y_mode else None,
                                            a_kind=pg.PRECOG_A_POWER),
-                            off, T, states_out=states, layer0=layer, L_total=shape.n_layers,
+                            off, T, states_out=states, layer0=slot, L_total=L_bank,
                             y_out=y)
     assert pg.precog_device_status()[0] == 0
+    assert bool(torch.isfinite(states[:, slot]).all()), "an entry of the written layer was not written"
+    assert bool(torch.isnan(states[:, :slot]).all()) and bool(torch.isnan(states[:, slot + 1:]).all()), \
+        "another layer was written"
     A = inp["A"].cpu().numpy()
+    ref = _oracle_states(inp["x"], inp["dt"], inp["B"], A, off_np, sample_chunks)
+    check = rel_err_stored if sdt == torch.bfloat16 else rel_err
     worst = 0.0
-    for c in sample_chunks:
-        s, e = int(off_np[c]), int(off_np[c + 1])
-        xs = to_np(inp["x"][s:e])
-        dts = to_np(inp["dt"][s:e])
-        Bs = to_np(inp["B"][s:e])
-        Cs = to_np(inp["C"][s:e]) if y_mode else None
-        ref_h, ref_y = oracle.rollout(xs, dts, A, Bs, Cs, want_y=y_mode)
-        err = rel_err_stored(to_np(states[c, layer]), ref_h)
+    for i, c in enumerate(sample_chunks):
+        err = check(to_np(states[c, slot]), ref[i])
         worst = max(worst, err)
         assert err < TOL_BF16, (c, err)
-        if y_mode:
-            assert rel_err_stored(to_np(y[0, s:e]), ref_y) < TOL_BF16
+    if y_mode:
+        for c in sample_chunks[:3]:
+            s, e = int(off_np[c]), int(off_np[c + 1])
+            _, ref_y = oracle.rollout(to_np(inp["x"][s:e]), to_np(inp["dt"][s:e]), A, to_np(inp["B"][s:e]),
+                                      to_np(inp["C"][s:e]), want_y=True)
+            assert rel_err_stored(to_np(y[0, s:e]), ref_y) < TOL_BF16, c
     del inp, states, y
     torch.cuda.empty_cache()
     return worst
@@ -317,7 +346,9 @@ def _sampled_check(dev, shape, layer, sample_chunks, y_mode=False, seed=0):
 def test_paper_shaped_multi_layer_call_sampled(cuda_device):
     """The launch the benchmark times: one call encodes 4 paper-shaped layers (4096 chunks x
     3000 tokens each, contiguous inputs of 4 independent draws) into layers 8..11 of the
-    24-layer bf16 bank; sampled chunks of every layer vs the oracle, other layers untouched."""
+    24-layer bf16 bank filled with NaN: every entry of those layers written and finite, the
+    other layers untouched, and per layer 36 seeded chunks (last wave included) vs the
+    oracle."""
     import torch
     pg = _pg()
     d = cuda_device
@@ -330,38 +361,47 @@ def test_paper_shaped_multi_layer_call_sampled(cuda_device):
     sets = [synth.device_scan_inputs(T, shape.D, shape.N, 0, l, d, with_C=False,
                                      out={"x": x[l], "dt": dt[l], "B": B[l]}) for l in range(S)]
     A = torch.stack([st["A"] for st in sets]).contiguous()
-    states = torch.full((shape.n_chunks, shape.n_layers, shape.D, shape.N), 5.0, dtype=torch.bfloat16,
-                        device=d)
+    states = torch.full((shape.n_chunks, shape.n_layers, shape.D, shape.N), float("nan"),
+                        dtype=torch.bfloat16, device=d)
     pg.precog_encode_chunks(pg.scan_inputs(x, dt, B, A, a_kind=pg.PRECOG_A_POWER),
                             torch.from_numpy(off_np).to(d), T, states_out=states, layer0=layer0,
                             L_total=shape.n_layers)
     assert pg.precog_device_status()[0] == 0
-    assert bool(torch.all(states[:, :layer0] == 5.0)) and bool(torch.all(states[:, layer0 + S:] == 5.0))
+    assert bool(torch.isnan(states[:, :layer0]).all()) and bool(torch.isnan(states[:, layer0 + S:]).all())
+    assert bool(torch.isfinite(states[:, layer0:layer0 + S]).all())
     An = sets[0]["A"].cpu().numpy()
     for l in range(S):
-        for c in (0, 2047, shape.n_chunks - 1):
-            sl = slice(int(off_np[c]), int(off_np[c + 1]))
-            ref_h, _ = oracle.rollout(to_np(x[l, sl]), to_np(dt[l, sl]), An, to_np(B[l, sl]))
-            assert rel_err_stored(to_np(states[c, layer0 + l]), ref_h) < TOL_BF16, (l, c)
+        pick = _sample(shape.n_chunks, (0, 2047, shape.n_chunks - 1), seed=l)
+        ref = _oracle_states(x[l], dt[l], B[l], An, off_np, pick)
+        for i, c in enumerate(pick):
+            assert rel_err_stored(to_np(states[c, layer0 + l]), ref[i]) < TOL_BF16, (l, c)
 
 
 def test_wide_single_layer_full_size(cuda_device):
-    """1 layer, D=2048, N=16, 1024 chunks x 512 tokens, bf16 (capture and y modes)."""
-    _sampled_check(cuda_device, synth.WIDE, 0, [0, 511, 1023])
-    _sampled_check(cuda_device, synth.WIDE, 0, [3, 1000], y_mode=True)
+    """1 layer, D=2048, N=16, 1024 chunks x 512 tokens, bf16: fp32 state capture (plain
+    tolerance) and the readout mode into a bf16 bank."""
+    _sampled_check(cuda_device, synth.WIDE, 0, _sample(1024, [0, 511, 1023]), state_dtype=_f32())
+    _sampled_check(cuda_device, synth.WIDE, 0, _sample(1024, [3, 1000], count=8, seed=1), y_mode=True)
+
+
+def _f32():
+    import torch
+    return torch.float32
 
 
 def test_paper_shaped_encode_full_size(cuda_device):
     """24 x (D=256, N=16) layers, 4096 chunks x 3000 tokens, bf16: layers 0 and 23 at
-    full size into the 192 KB-per-chunk bf16 bank layout."""
-    _sampled_check(cuda_device, synth.PAPER, 0, [0, 2047, 4095])
-    _sampled_check(cuda_device, synth.PAPER, 23, [1, 4094])
+    full size into the 192 KB-per-chunk bf16 bank layout, and layer 5 captured in fp32
+    (plain tolerance, no rounding allowance)."""
+    _sampled_check(cuda_device, synth.PAPER, 0, _sample(4096, [0, 2047, 4095]))
+    _sampled_check(cuda_device, synth.PAPER, 23, _sample(4096, [1, 4094], seed=23))
+    _sampled_check(cuda_device, synth.PAPER, 5, _sample(4096, [7], seed=5), state_dtype=_f32())
 
 
 def test_ragged_large_scale_encode_full_size(cuda_device):
     """8192 ragged chunks (lengths 256..4096), D=512, N=16, bf16: the longest, the
-    shortest and a few random chunks of one layer."""
+    shortest, the first and last and 36 seeded chunks of one layer."""
     off = synth.shape_offsets(synth.RAGGED, 0)
     lens = np.diff(off)
-    pick = sorted({int(np.argmax(lens)), int(np.argmin(lens)), 0, 4097, 8191})
-    _sampled_check(cuda_device, synth.RAGGED, 5, pick)
+    fixed = [int(np.argmax(lens)), int(np.argmin(lens)), 0, 4097, 8191]
+    _sampled_check(cuda_device, synth.RAGGED, 5, _sample(8192, fixed, seed=5))

@@ -31,8 +31,8 @@ def _topk(index, queries, k):
                                        (4099, 9, 8, 64), (20000, 200, 5, 136), (300, 300, 2, 64)])
 def test_topk_exact_integer_scores(cuda_device, dtype_name, M, Q, k, dim):
     """Small-integer keys: exact scores, many ties. Rows and scores must equal the
-    oracle's stable ranking bit for bit, on the CUDA-core path (Q = 1, or fp32) and
-    the tensor-core path (fp16/bf16, Q >= 2)."""
+    oracle's stable ranking bit for bit, on the CUDA-core path (fp32 keys) and the
+    tensor-core path (fp16/bf16 keys, any batch)."""
     import torch
     dtype = getattr(torch, dtype_name)
     if dtype == torch.float32 and Q > 50:
@@ -132,3 +132,13 @@ def test_retrieve_topk_then_compose_query_workload(cuda_device):
                                           to_np(C[l, sl]), h0=h0, want_y=True)
             assert rel_err_stored(to_np(h[q, l]), ref_h) < TOL_BF16
             assert rel_err_stored(to_np(y[l, sl]), ref_y) < TOL_BF16
+
+
+@pytest.mark.parametrize("dtype_name", ["float16", "float32"])
+def test_topk_empty_index(cuda_device, dtype_name):
+    """No rows: every entry of every query's list is row -1 with a NaN score."""
+    import torch
+    dtype = getattr(torch, dtype_name)
+    idx, score = _topk(torch.empty((0, 64), dtype=dtype, device=cuda_device),
+                       torch.ones((2, 64), dtype=dtype, device=cuda_device), 3)
+    assert (idx == -1).all() and np.isnan(score).all()
