@@ -707,13 +707,26 @@ def main():
     scan_in = [pg.scan_inputs(st["x"], st["dt"], st["B"], st["A"], a_kind=pg.PRECOG_A_POWER) for st in sets]
     calls = L // S
 
-    # query-time workload
+    # query-time workload. One rank: the whole index and bank. Several ranks: the index
+    # and the bank are sharded by rows (each rank holds M / world of each); every rank
+    # serves the same queries, retrieving over its rows, combining the shards' keys with
+    # one all-reduce MAX and receiving the winning states from their owners (an all-reduce
+    # of owner-filled rows) before it prefills.
     M, dim, Tq, Q = synth.QUERY_INDEX_M, synth.QUERY_DIM, synth.QUERY_TOKENS, args.query_batch
-    index = synth.device_unit_index(M, dim, seed + 1, dev)
-    qbank = synth.device_normal_bank(M, L * D * N, seed + 2, dev).view(M, L, D, N)
+    qseed0 = 1 if world > 1 else seed          # the same index and queries on every rank
+    index_full = synth.device_unit_index(M, dim, qseed0 + 1, dev)
+    if world > 1:
+        from paper_2608_02560_gb300 import distributed as pgd
+        row_off, rows_here = pgd.shard_rows(M, world, rank)
+        index = index_full[row_off:row_off + rows_here].clone()
+        qbank = synth.device_normal_bank(rows_here, L * D * N, 2 + 1000 * rank, dev).view(rows_here, L, D, N)
+    else:
+        row_off, rows_here = 0, M
+        index = index_full
+        qbank = synth.device_normal_bank(M, L * D * N, seed + 2, dev).view(M, L, D, N)
 
     def query_batch(nq, qseed):
-        q, rows = synth.device_planted_queries(index, nq, synth.QUERY_NOISE, qseed)
+        q, rows = synth.device_planted_queries(index_full, nq, synth.QUERY_NOISE, qseed)
         ins = [synth.device_scan_inputs(nq * Tq, D, N, qseed, l, dev) for l in range(L)]
         st = lambda k: torch.stack([i[k] for i in ins]).contiguous()
         qx, qdt, qB, qC, qA = st("x"), st("dt"), st("B"), st("C"), st("A")
@@ -721,15 +734,23 @@ def main():
                "in": pg.scan_inputs(qx, qdt, qB, qA, qC, a_kind=pg.PRECOG_A_POWER),
                "idx": torch.empty(nq, dtype=torch.int64, device=dev),
                "score": torch.empty(nq, dtype=torch.float32, device=dev),
-               "ws": torch.empty(pg.precog_retrieve_workspace_size(M, dim, nq) + 16,
+               "ws": torch.empty(pg.precog_retrieve_workspace_size(rows_here, dim, nq) + 16,
                                  dtype=torch.uint8, device=dev),
+               "inj": torch.empty((nq, L, D, N), dtype=torch.bfloat16, device=dev) if world > 1 else None,
                "y": torch.empty((L, nq * Tq, D), dtype=torch.bfloat16, device=dev),
                "h": torch.empty((nq, L, D, N), dtype=torch.bfloat16, device=dev), "n": nq}
         return out
 
-    qb = query_batch(Q, seed + 3)
+    qb = query_batch(Q, qseed0 + 3)
 
     def query_path(b, stream=None):
+        if world > 1:
+            # torch's current stream carries the kernels and the collectives
+            pgd.sharded_retrieve(index, b["q"], row_off, b["idx"], b["score"], workspace=b["ws"])
+            pgd.gather_owned_states(qbank, row_off, b["idx"], b["inj"])
+            pg.precog_prefill_from_state(b["in"], b["n"], Tq, b["inj"], idx=None, y_out=b["y"],
+                                         state_out=b["h"])
+            return
         pg.precog_retrieve(index, b["q"], b["idx"], b["score"], workspace=b["ws"], stream=stream)
         pg.precog_prefill_from_state(b["in"], b["n"], Tq, qbank, idx=b["idx"], y_out=b["y"],
                                      state_out=b["h"], stream=stream)
@@ -906,31 +927,36 @@ def main():
             return times[len(times) // 2], times[int(len(times) * 0.9)]
 
         for nq, iters in ((1, args.latency_iters), (256, max(20, args.latency_iters // 4))):
-            b = qb if nq == Q else query_batch(nq, seed + 7 + nq)
+            b = qb if nq == Q else query_batch(nq, qseed0 + 7 + nq)
             for _ in range(3):
                 query_path(b)
             p50, p90 = p50_p90(lambda: query_path(b), iters)
-            side = torch.cuda.Stream()
-            side.wait_stream(torch.cuda.current_stream())
-            with torch.cuda.stream(side):
-                query_path(b)
-            torch.cuda.current_stream().wait_stream(side)
-            graph = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(graph):
-                query_path(b)
-            g50, _ = p50_p90(graph.replay, iters)
+            g50 = None
+            if world == 1:
+                side = torch.cuda.Stream()
+                side.wait_stream(torch.cuda.current_stream())
+                with torch.cuda.stream(side):
+                    query_path(b)
+                torch.cuda.current_stream().wait_stream(side)
+                graph = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(graph):
+                    query_path(b)
+                g50, _ = p50_p90(graph.replay, iters)
+                del graph
             # the index sweep alone, at the measured copy bandwidth, bounds the latency below
-            floor_us = M * dim * index.element_size() / (peaks()[0] * 1e9) * 1e6
+            floor_us = rows_here * dim * index.element_size() / (peaks()[0] * 1e9) * 1e6
             latency[f"q{nq}"] = {"p50_us": p50, "p90_us": p90, "iters": iters,
                                  "graph_p50_us": g50, "index_sweep_floor_us": floor_us,
                                  "retrieved_planted": bool(torch.equal(b["idx"], b["rows"]))}
-            del graph
+            if world > 1:
+                latency[f"q{nq}"]["index_rows_per_rank"] = rows_here
             if b is not qb:
                 del b
         del flush, evict
 
+    # the extension rows and the other configurations are single-GPU measurements
     extras = None
-    if not args.no_extras:
+    if not args.no_extras and world == 1:
         extras = measure_extensions(pg, synth, torch, dev, sets[0], off, T, shape.n_chunks, index, qbank,
                                     query_batch, peaks()[0], call_in=call_in, layers_per_call=S)
 
@@ -958,8 +984,8 @@ def main():
 
     # ---------------- the other encode configurations, on their own resident inputs
     configs = None
-    if not args.no_configs:
-        del x_all, dt_all, B_all, sets, call_in, scan_in, qbank, index, bank, qb
+    if not args.no_configs and world == 1:
+        del x_all, dt_all, B_all, sets, call_in, scan_in, qbank, index, index_full, bank, qb
         torch.cuda.empty_cache()
         alu_peak_v = alu_peak_tops(dev)[0]
         configs, cfg_samples = measure_configs(pg, synth, torch, dev, peaks()[0], alu_peak_v, n_cpu)
@@ -986,6 +1012,9 @@ def main():
                            "input_sets_resident": S, "layers_per_encode_call": S,
                            "index_rows": M, "index_dim": dim, "bank_entries": M,
                            "query_batch": Q, "query_tokens": Tq, "parallelism": f"dp{world}",
+                           "query_path": ("index and bank rows sharded over the ranks; one all-reduce MAX of "
+                                          "the shards' keys, the winning states gathered by an all-reduce of "
+                                          "owner-filled rows") if world > 1 else "whole index and bank on one GPU",
                            "l2": "inputs larger than L2 (12.98 GB per layer, 1.5 GB index)"},
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks,
                 "gpu_launches": int(launches), "latency": latency,

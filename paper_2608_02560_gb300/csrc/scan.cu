@@ -5,8 +5,10 @@
 // thread owns CPT adjacent channels and keeps their N = 16 fp32 states in
 // registers for the whole chunk. The chunk's rows of x and dt (DS channels
 // each) and of B (and C) are staged into shared memory TILE tokens at a time
-// by the TMA engine (1-D bulk copies completing on an mbarrier), in a
-// STAGES-deep ring, so the time loop only reads shared memory.
+// by the TMA engine, completing on an mbarrier, in a STAGES-deep ring, so the
+// time loop only reads shared memory: a whole-row slice is one contiguous 1-D
+// bulk copy per tensor; a narrower slice (rows wider than 512 channels) is one
+// tiled tensor-map copy of TILE rows per tensor.
 //
 // Per token and channel the recurrence is, for the 16 state indices n,
 //   h[n] <- alpha_n * h[n] + (dt * x) * B[n],   alpha_n = exp(dt * A[d, n]).
@@ -103,6 +105,14 @@ struct Cfg {
 struct TrajCursor {
     int64_t entry;
     int64_t left;
+};
+
+// Tensor maps of x and dt for launches whose CTAs take a slice of each row: the tensor is
+// viewed as [layer][row][D / inner][inner] (inner = min(slice, 256) channels, the widest
+// box dimension), so a box of [1][TILE][slice / inner][inner] is one slice of TILE rows.
+struct SliceMaps {
+    CUtensorMap x, dt;
+    int32_t valid, inner;
 };
 
 struct StageLayout {
@@ -602,7 +612,7 @@ __device__ __forceinline__ void scan_tile_rescaled(const unsigned char *st, cons
 // ---------------------------------------------------------------------------
 template <class C>
 __global__ void __launch_bounds__(C::LB_THREADS, C::LB_BLOCKS)
-    scan_kernel(const ScanParams p, const int DS_arg, const int slices) {
+    scan_kernel(const ScanParams p, const int DS_arg, const int slices, const __grid_constant__ SliceMaps maps) {
     using TIn = typename C::TIn;
     const int DS = C::FIXDS ? C::FIXDS : DS_arg;
     constexpr int CPT = C::CPT, TILE = C::TILE, STAGES = C::STAGES, SZ = C::SZ;
@@ -694,11 +704,18 @@ __global__ void __launch_bounds__(C::LB_THREADS, C::LB_BLOCKS)
         const int ntok = static_cast<int>(min64(TILE, len - k * TILE));
         const uint32_t rowb = DS * SZ;
         const uint32_t bytes = ntok * rowb * 2 + ntok * kN * SZ * (C::HAS_Y ? 2 : 1);
-        mbar_arrive_expect_tx(&full[s], bytes);
         if (DS == D) {
+            mbar_arrive_expect_tx(&full[s], bytes);
             bulk_g2s(st + lay.xs, xl + row0 * D, ntok * rowb, &full[s]);
             bulk_g2s(st + lay.dts, dtl + row0 * D, ntok * rowb, &full[s]);
+        } else if (maps.valid) {
+            // the slice of TILE rows as one tensor-map copy per tensor (a box always moves
+            // TILE rows; rows past the end of the tensor arrive as zeros)
+            mbar_arrive_expect_tx(&full[s], bytes + (TILE - ntok) * rowb * 2);
+            tma_load_4d(st + lay.xs, &maps.x, 0, d0 / maps.inner, static_cast<int32_t>(row0), layer, &full[s]);
+            tma_load_4d(st + lay.dts, &maps.dt, 0, d0 / maps.inner, static_cast<int32_t>(row0), layer, &full[s]);
         } else {
+            mbar_arrive_expect_tx(&full[s], bytes);
             for (int r = 0; r < ntok; ++r) {
                 bulk_g2s(st + lay.xs + r * rowb, xl + (row0 + r) * D + d0, rowb, &full[s]);
                 bulk_g2s(st + lay.dts + r * rowb, dtl + (row0 + r) * D + d0, rowb, &full[s]);
@@ -893,18 +910,35 @@ bool few_items(const ScanParams &p) {
 
 template <class C>
 cudaError_t launch_cfg(const ScanParams &p, cudaStream_t stream) {
-    const int DS = pick_slice(p.D, C::SZ, C::CPT, C::MAXSLICE);
-    if (DS == 0 || (C::FIXDS && DS != C::FIXDS)) return cudaErrorInvalidValue;
+    const int DS = C::FIXDS ? (p.D % C::FIXDS == 0 && (C::FIXDS * C::SZ) % 16 == 0 ? C::FIXDS : 0)
+                            : pick_slice(p.D, C::SZ, C::CPT, C::MAXSLICE);
+    if (DS == 0) return cudaErrorInvalidValue;
     const int slices = p.D / DS;
     const StageLayout lay = stage_layout(C::TILE, DS, C::SZ, C::HAS_Y, C::CONV);
     const size_t smem = kBarBytes + static_cast<size_t>(C::STAGES) * lay.bytes;
     const int64_t items = static_cast<int64_t>(p.n_layers) * p.n_chunks * slices;
     if (items == 0) return cudaSuccess;
     if (items > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+    SliceMaps maps{};
+    if (DS < p.D) {
+        const int inner = DS < 256 ? DS : 256;
+        const cuuint64_t rows = static_cast<cuuint64_t>(p.T_tot);
+        const cuuint64_t dims[4] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(p.D / inner), rows,
+                                    static_cast<cuuint64_t>(p.n_layers)};
+        const cuuint64_t lstride = static_cast<cuuint64_t>(p.n_layers > 1 ? p.ls_xd : rows * p.D) * C::SZ;
+        const cuuint64_t strides[3] = {static_cast<cuuint64_t>(inner) * C::SZ, static_cast<cuuint64_t>(p.D) * C::SZ,
+                                       lstride};
+        const cuuint32_t box[4] = {static_cast<cuuint32_t>(inner), static_cast<cuuint32_t>(DS / inner),
+                                   static_cast<cuuint32_t>(C::TILE), 1};
+        const CUtensorMapDataType dt = C::SZ == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+        maps.valid = encode_tiled_map(&maps.x, dt, 4, p.x, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_NONE) &&
+                     encode_tiled_map(&maps.dt, dt, 4, p.dt, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_NONE);
+        maps.inner = inner;
+    }
     auto kern = scan_kernel<C>;
     cudaError_t e = ensure_smem(reinterpret_cast<const void *>(kern), static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    kern<<<static_cast<unsigned>(items), DS / C::CPT, smem, stream>>>(p, DS, slices);
+    kern<<<static_cast<unsigned>(items), DS / C::CPT, smem, stream>>>(p, DS, slices, maps);
     e = cudaGetLastError();
     if (e == cudaSuccess) count_launches(1);
     return e;
@@ -925,14 +959,19 @@ cudaError_t launch_t(const ScanParams &p, cudaStream_t stream) {
         else
             return launch_cfg<Cfg<TIn, false, false, MODE, 2, 16, 4, 3, kTrajDirect>>(p, stream);
     } else if constexpr (MODE == kPower && !HAS_Y) {
-        // the corpus encode of 256-channel rows (the paper's layer width) gets a slice fixed
-        // at compile time
-        if constexpr (!HAS_H0 && !std::is_same<TIn, float>::value)
-            if (pick_slice(p.D, sizeof(TIn), PRECOG_RESCALED_CPT, kWideSlice) == 256) {
-                using C256 = Cfg<TIn, false, false, MODE, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
-                                 PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB, kTrajNone, kWideSlice, 256>;
-                return launch_cfg<C256>(p, stream);
-            }
+        // the corpus encode of 256- and 512-channel slices (the paper's layer width, the
+        // ragged and wide workloads' slices) gets the slice fixed at compile time
+        if constexpr (!HAS_H0 && !std::is_same<TIn, float>::value) {
+            const int ds = pick_slice(p.D, sizeof(TIn), PRECOG_RESCALED_CPT, kWideSlice);
+            if (ds == 256)
+                return launch_cfg<Cfg<TIn, false, false, MODE, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
+                                      PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB, kTrajNone, kWideSlice, 256>>(
+                    p, stream);
+            if (ds == 512)
+                return launch_cfg<Cfg<TIn, false, false, MODE, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
+                                      PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB, kTrajNone, kWideSlice, 512>>(
+                    p, stream);
+        }
         return launch_cfg<Cfg<TIn, HAS_Y, HAS_H0, MODE, PRECOG_RESCALED_CPT, PRECOG_RESCALED_TILE,
                               PRECOG_RESCALED_STAGES, PRECOG_RESCALED_MINB, kTrajNone, kWideSlice>>(p, stream);
     } else {

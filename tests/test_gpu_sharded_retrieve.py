@@ -64,3 +64,37 @@ def test_empty_shard_and_no_row_keys(cuda_device):
     sc = torch.empty(3, dtype=torch.float32, device=d)
     pg.precog_decode_keys(k, idx, sc)
     assert torch.all(idx == -1) and torch.all(torch.isnan(sc))
+
+
+def test_sharded_query_path_equals_whole_bank_injection(cuda_device):
+    """The sharded query path of several ranks, emulated on one GPU: every shard of the
+    bank contributes its owned winning rows (gather_owned_states without a process group),
+    the sum over shards is the all-reduce the ranks run, and prefilling from those gathered
+    states (no index) gives exactly the y and states of injecting from the whole bank."""
+    import torch
+    import paper_2608_02560_gb300 as pg
+    from paper_2608_02560_gb300.distributed import gather_owned_states, shard_rows
+    d = cuda_device
+    M, L, D, N, Tq, Q = 1000, 3, 64, 16, 20, 6
+    bank = synth.device_normal_bank(M, L * D * N, 4, d).view(M, L, D, N)
+    idx = torch.tensor([0, 999, 333, -1, 334, 333], dtype=torch.int64, device=d)
+    ins = [synth.device_scan_inputs(Q * Tq, D, N, 9, l, d) for l in range(L)]
+    st = lambda k: torch.stack([i[k] for i in ins]).contiguous()
+    si = pg.scan_inputs(st("x"), st("dt"), st("B"), st("A"), st("C"), a_kind=pg.PRECOG_A_POWER)
+    y_ref = torch.empty((L, Q * Tq, D), dtype=torch.bfloat16, device=d)
+    h_ref = torch.empty((Q, L, D, N), dtype=torch.bfloat16, device=d)
+    pg.precog_prefill_from_state(si, Q, Tq, bank, idx=idx, y_out=y_ref, state_out=h_ref)
+    world = 3
+    total = torch.zeros((Q, L, D, N), dtype=torch.float32, device=d)
+    for r in range(world):
+        off, rows = shard_rows(M, world, r)
+        part = torch.empty((Q, L, D, N), dtype=torch.bfloat16, device=d)
+        gather_owned_states(bank[off:off + rows], off, idx, part)
+        total += part.float()
+    inj = total.to(torch.bfloat16)
+    assert torch.equal(inj[3], torch.zeros_like(inj[3])) and torch.equal(inj[0], bank[0])
+    y = torch.empty_like(y_ref)
+    h = torch.empty_like(h_ref)
+    pg.precog_prefill_from_state(si, Q, Tq, inj, idx=None, y_out=y, state_out=h)
+    assert pg.precog_device_status()[0] == 0
+    assert torch.equal(y, y_ref) and torch.equal(h, h_ref)

@@ -136,3 +136,46 @@ def test_shard_rows_tile_the_index(M, world):
     assert pos == M
     sizes = [rows for _, rows in blocks]
     assert max(sizes) - min(sizes) <= 1
+
+
+def _gather_main(rank, world, port, queue):
+    import torch
+    import torch.distributed as dist
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        from paper_2608_02560_gb300.distributed import gather_owned_states, shard_rows
+        M, L, E = 11, 2, 6
+        bank = torch.arange(M * L * E, dtype=torch.float32).view(M, L, E) - 20.0
+        bank[4, 1, 2] = float("nan")
+        off, rows = shard_rows(M, world, rank)
+        idx = torch.tensor([0, 10, 5, -1, 4, 5, 6], dtype=torch.int64)
+        out = torch.full((idx.numel(), L, E), 7.0)
+        gather_owned_states(bank[off:off + rows].clone(), off, idx, out)
+        queue.put((rank, out.numpy().tolist()))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_gloo_ranks_gather_owned_states():
+    """Sharded injection: every rank ends with the global bank rows its queries won (rows
+    owned by either rank, a repeated row, a NaN entry), and row -1 gives the zero state."""
+    import numpy as np
+    import torch
+    mp = pytest.importorskip("torch.multiprocessing")
+    ctx = mp.get_context("spawn")
+    queue = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_gather_main, args=(r, 2, port, queue)) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(timeout=180)
+    assert all(p.exitcode == 0 for p in procs), [p.exitcode for p in procs]
+    res = sorted(queue.get(timeout=10) for _ in range(2))
+    bank = torch.arange(11 * 2 * 6, dtype=torch.float32).view(11, 2, 6) - 20.0
+    bank[4, 1, 2] = float("nan")
+    want = torch.stack([bank[i] if i >= 0 else torch.zeros(2, 6) for i in (0, 10, 5, -1, 4, 5, 6)]).numpy()
+    for _, got in res:
+        np.testing.assert_array_equal(np.array(got), want)
