@@ -821,7 +821,17 @@ __global__ void __launch_bounds__(C::LB_THREADS, C::LB_BLOCKS)
         if (C::CONV && ok) {
             const TIn *bsrc = reinterpret_cast<const TIn *>(st + lay.bs);
             float *bdst = reinterpret_cast<float *>(st + lay.bf);
-            for (int i = tid; i < ntok * kN; i += nthr) bdst[i] = to_f32(bsrc[i]);
+            if constexpr (std::is_same<TIn, __nv_bfloat16>::value) {
+                // four values per thread and step: one 8-byte read, one 16-byte write
+                for (int i = tid * 4; i < ntok * kN; i += nthr * 4) {
+                    const uint2 w = *reinterpret_cast<const uint2 *>(bsrc + i);
+                    *reinterpret_cast<float4 *>(bdst + i) =
+                        make_float4(__uint_as_float(w.x << 16), __uint_as_float(w.x & 0xffff0000u),
+                                    __uint_as_float(w.y << 16), __uint_as_float(w.y & 0xffff0000u));
+                }
+            } else {
+                for (int i = tid; i < ntok * kN; i += nthr) bdst[i] = to_f32(bsrc[i]);
+            }
             if (C::HAS_Y) {
                 const TIn *csrc = reinterpret_cast<const TIn *>(st + lay.cs);
                 float *cdst = reinterpret_cast<float *>(st + lay.cf);
