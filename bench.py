@@ -615,7 +615,7 @@ def cpu_baseline(oracle, paper, others, query, L):
 
     res = {"kind": "oracle", "unit": UNIT, "cores": cores}
     one, s1, tok1 = rate(paper, 1, 16)
-    n_all = min(paper["offsets"].shape[0] - 1, 4 * cores)
+    n_all = paper["offsets"].shape[0] - 1
     allc, sa, toka = rate(paper, cores, n_all)
     res.update(value=allc, seconds=sa,
                sample=f"{n_all} chunks x 3000 tokens x 1 layer of the paper-shaped encode on {cores} host "
@@ -624,10 +624,11 @@ def cpu_baseline(oracle, paper, others, query, L):
                single_core={"value": one, "seconds": s1, "sample": "16 chunks x 3000 tokens x 1 layer, one core"})
     for name, smp in others.items():
         n = smp["offsets"].shape[0] - 1
-        o1, t1, _ = rate(smp, 1, n)
+        o1, t1, _ = rate(smp, 1, min(n, 16))
         oa, ta, _ = rate(smp, cores, n)
         res[name] = {"single_core": o1, "all_cores": oa, "seconds": [t1, ta],
-                     "sample": f"{n} chunks x 1 layer, rate divided by {smp['layers']} layer(s)"}
+                     "sample": f"{min(n, 16)} chunks x 1 layer on one core, {n} chunks x 1 layer on "
+                               f"{cores} threads; rates divided by {smp['layers']} layer(s)"}
     if query is not None:
         t0 = time.perf_counter()
         idx, _ = oracle.retrieve(query["index"], query["q"])
@@ -970,7 +971,7 @@ def main():
     cpu_paper = cpu_query = None
     n_cpu = 16
     if want_cpu:
-        n_paper = max(n_cpu, 4 * (os.cpu_count() or 1))
+        n_paper = max(n_cpu, 16 * (os.cpu_count() or 1))
         r1 = n_paper * shape.chunk_len
         cpu_paper = {k: sets[0][k][:r1].cpu().double().numpy() for k in ("x", "dt", "B")}
         cpu_paper.update(A=sets[0]["A"].cpu().double().numpy(), offsets=synth.fixed_offsets(n_paper, shape.chunk_len),
@@ -988,7 +989,8 @@ def main():
         del x_all, dt_all, B_all, sets, call_in, scan_in, qbank, index, index_full, bank, qb
         torch.cuda.empty_cache()
         alu_peak_v = alu_peak_tops(dev)[0]
-        configs, cfg_samples = measure_configs(pg, synth, torch, dev, peaks()[0], alu_peak_v, n_cpu)
+        configs, cfg_samples = measure_configs(pg, synth, torch, dev, peaks()[0], alu_peak_v,
+                                               max(n_cpu, 4 * (os.cpu_count() or 1)))
         st, bits = pg.precog_device_status()
         if st != 0:
             raise RuntimeError(f"device status {st} bits {bits:#x} after the configuration runs")
