@@ -141,22 +141,32 @@ def test_multi_layer_call_and_layer_offset(cuda_device):
             assert rel_err(got[c, 2 + l], ref[c]) < TOL_F32
 
 
-@pytest.mark.parametrize("D,y_mode", [(512, False), (1024, False), (768, False), (4096, False),
-                                      (1024, True), (768, True)])
-def test_multi_layer_sliced_channels(cuda_device, D, y_mode):
+@pytest.mark.parametrize("D,y_mode,dtype_name", [(512, False, "float32"), (1024, False, "float32"),
+                                                 (768, False, "float32"), (4096, False, "float32"),
+                                                 (1024, True, "float32"), (768, True, "float32"),
+                                                 (1024, False, "bfloat16"), (2048, True, "bfloat16"),
+                                                 (768, False, "bfloat16")])
+def test_multi_layer_sliced_channels(cuda_device, D, y_mode, dtype_name):
     """Rows wider than one CTA's channel slice (512 channels with the power-form A, 256
-    where 512 does not divide D: 2, 3 and 8 slices here), three layers in one call: each
-    CTA stages its slice of every x and dt row with one bulk copy per row; D = 512 stays
-    one slice. Chunks (one of them empty) end inside and at the end of 16-row tiles.
-    Every layer's states (and y) vs the oracle."""
+    where 512 does not divide D: 2, 3, 4 and 8 slices here), three layers in one call: each
+    CTA stages its slice of TILE rows of x and dt with one tensor-map copy per tensor (a box
+    that reaches past the last row arrives zero-filled); D = 512 stays one slice. Chunks
+    (one of them empty) end inside and at the end of 16-row tiles. fp32 and bf16 inputs
+    (the bf16 values widened exactly for the oracle). Every layer's states (and y) vs the
+    oracle."""
     import torch
     pg = _pg()
     d = cuda_device
+    dtype = getattr(torch, dtype_name)
     L, N = 3, 16
     off = np.array([0, 1, 17, 17, 53, 200], dtype=np.int64)
     T = int(off[-1])
     ins = [synth.host_scan_inputs(T, D, N, seed=90 + l) for l in range(L)]
-    st = lambda k: _t(np.stack([i[k] for i in ins]), d)
+    if dtype == torch.bfloat16:
+        # the values the kernel sees: rounded to bf16 once, exactly representable in fp64
+        ins = [tuple(a if i == 2 else torch.from_numpy(np.ascontiguousarray(a)).to(torch.bfloat16).double().numpy()
+                     for i, a in enumerate(t)) for t in ins]
+    st = lambda k: _t(np.stack([i[k] for i in ins]), d, dtype)
     x, dt, B, C = st(0), st(1), st(3), st(4)
     A = _t(np.stack([synth.structured_A(D, N) * (1 + 0.25 * l) for l in range(L)]), d)
     n = len(off) - 1
@@ -169,13 +179,14 @@ def test_multi_layer_sliced_channels(cuda_device, D, y_mode):
     for l in range(L):
         ref, ref_y = oracle.scan(ins[l][0], ins[l][1], synth.structured_A(D, N) * (1 + 0.25 * l),
                                  ins[l][3], off, C=ins[l][4] if y_mode else None, want_y=y_mode)
+        tol = TOL_F32 if dtype == torch.float32 else TOL_BF16
         for c in range(n):
             if off[c] == off[c + 1]:
                 assert np.all(got[c, l] == 0)
             else:
-                assert rel_err(got[c, l], ref[c]) < TOL_F32
+                assert rel_err(got[c, l], ref[c]) < tol
         if y_mode:
-            assert rel_err(to_np(y[l]), ref_y) < TOL_F32
+            assert rel_err(to_np(y[l]), ref_y) < tol
 
 
 def test_bf16_capture_and_readout(cuda_device):
