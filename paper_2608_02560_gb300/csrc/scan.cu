@@ -684,6 +684,25 @@ __global__ void __launch_bounds__(C::LB_THREADS, C::LB_BLOCKS)
     item /= slices;
     const int64_t chunk = item % p.n_chunks;
     const int layer = static_cast<int>(item / p.n_chunks);
+    // this thread's rows of A first (16 floats each, 16-byte loads): their latency overlaps
+    // the chunk's offsets below
+    float a_rows[CPT][kN];
+    {
+        const float *Al0 = p.A + static_cast<int64_t>(layer) * p.D * kN;
+#pragma unroll
+        for (int j = 0; j < CPT; ++j) {
+            const float4 *a4 = reinterpret_cast<const float4 *>(
+                Al0 + static_cast<int64_t>(slice * DS + static_cast<int>(threadIdx.x) * CPT + j) * kN);
+#pragma unroll
+            for (int q = 0; q < kN / 4; ++q) {
+                const float4 v = a4[q];
+                a_rows[j][4 * q] = v.x;
+                a_rows[j][4 * q + 1] = v.y;
+                a_rows[j][4 * q + 2] = v.z;
+                a_rows[j][4 * q + 3] = v.w;
+            }
+        }
+    }
     int64_t start, len;
     if (p.use_fixed) {
         start = chunk * p.fixed_len;
@@ -715,31 +734,26 @@ __global__ void __launch_bounds__(C::LB_THREADS, C::LB_BLOCKS)
     const TIn *dtl = static_cast<const TIn *>(p.dt) + layer * p.ls_xd;
     const TIn *Bl = static_cast<const TIn *>(p.B) + layer * p.ls_bc;
     const TIn *Cl = C::HAS_Y ? static_cast<const TIn *>(p.C) + layer * p.ls_bc : nullptr;
-    const float *Al = p.A + static_cast<int64_t>(layer) * D * kN;
 
     // ---- coefficients; kPower verifies the structure (A[d, n] = (n + 1) A[d, 0] <= 0) ----
     float kpow[CPT];      // A[d, 0] * log2 e
     f2 kgen[CPT][8];      // (A[d, n] * log2 e) pairs, kGeneral only
+    bool a_ok = true;
 #pragma unroll
     for (int j = 0; j < CPT; ++j) {
-        const float *a = Al + static_cast<int64_t>(d0 + dl + j) * kN;
+        const float (&a)[kN] = a_rows[j];
         kpow[j] = a[0] * kLog2e;
         if constexpr (C::MODE == kGeneral) {
 #pragma unroll
             for (int i = 0; i < 8; ++i) kgen[j][i] = pack2(a[2 * i] * kLog2e, a[2 * i + 1] * kLog2e);
+        } else {
+            a_ok &= a[0] <= 0.f;
+#pragma unroll
+            for (int n = 1; n < kN; ++n) a_ok &= a[n] == static_cast<float>(n + 1) * a[0];
         }
     }
     if constexpr (C::MODE == kPower) {
-        bool ok = true;
-#pragma unroll
-        for (int j = 0; j < CPT; ++j) {
-            const float *a = Al + static_cast<int64_t>(d0 + dl + j) * kN;
-            const float a0 = a[0];
-            ok &= a0 <= 0.f;
-#pragma unroll
-            for (int n = 1; n < kN; ++n) ok &= a[n] == static_cast<float>(n + 1) * a0;
-        }
-        if (!__syncthreads_and(ok)) {
+        if (!__syncthreads_and(a_ok)) {
             if (tid == 0) atomicOr(&g_scan_status, PRECOG_DEV_BAD_A);
             return;
         }
