@@ -426,7 +426,9 @@ __global__ void __launch_bounds__(block_channels<HAS_Y>())
     const float a1 = Al[1].y, re0 = Al[0].x;
 #pragma unroll
     for (int i = 0; i < kP; ++i) {
-        const float2 q0 = Al[2 * i], q1 = Al[2 * i + 1];
+        // the pair of complex values 2i, 2i+1 in one 16-byte load
+        const float4 q = reinterpret_cast<const float4 *>(Al)[i];
+        const float2 q0 = make_float2(q.x, q.y), q1 = make_float2(q.z, q.w);
         ar[i] = pack2(q0.x * kLog2e, q1.x * kLog2e);
         ai[i] = pack2(q0.y, q1.y);
         nai[i] = pack2(-q0.y, -q1.y);

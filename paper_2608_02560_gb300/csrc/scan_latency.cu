@@ -124,11 +124,13 @@ __global__ void __launch_bounds__(kLThreads)
     // ---- the power statement, verified before anything is staged or written ----
     const float *a = p.A + (static_cast<int64_t>(layer) * D + d) * kN;
     const float a0 = a[0];
+    const float4 aq = *reinterpret_cast<const float4 *>(a + 4 * g);   // this thread's 4 values
+    const float av[4] = {aq.x, aq.y, aq.z, aq.w};
     bool ok = a0 <= 0.f;
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
         const int n = 4 * g + k;
-        ok &= a[n] == static_cast<float>(n + 1) * a0;
+        ok &= av[k] == static_cast<float>(n + 1) * a0;
     }
     const float kpow = a0 * kLog2e;
     const float coef = static_cast<float>(4 * g + 1);
