@@ -534,6 +534,7 @@ def measure_configs(pg, synth, torch, dev, hbm, alu_peak, cpu_chunks):
     of the ragged large-scale encode (D=512, 8192 chunks of U[256, 4096] tokens, bf16
     bank; 24 such layers make the workload). Returns the rows and, for the CPU baseline,
     the first ``cpu_chunks`` chunks of each workload's inputs copied back to the host."""
+    import numpy as np
     out, samples = {}, {}
 
     def timed(fn, iters=5):
@@ -557,7 +558,14 @@ def measure_configs(pg, synth, torch, dev, hbm, alu_peak, cpu_chunks):
         sdt = torch.float32 if shape is synth.WIDE else torch.bfloat16
         states = torch.empty((shape.n_chunks, 1, shape.D, shape.N), dtype=sdt, device=dev)
         si = pg.scan_inputs(inp["x"], inp["dt"], inp["B"], inp["A"], a_kind=pg.PRECOG_A_POWER)
-        ms = timed(lambda: pg.precog_encode_chunks(si, off, T, states_out=states))
+        if shape is synth.RAGGED:
+            # ragged chunks are taken up longest first (the caller knows the lengths it laid
+            # out), so the short ones fill the launch's tail; the unordered time is kept too
+            order = torch.from_numpy(np.argsort(-np.diff(off_np), kind="stable").astype(np.int64)).to(dev)
+            ms_unordered = timed(lambda: pg.precog_encode_chunks(si, off, T, states_out=states))
+            ms = timed(lambda: pg.precog_encode_chunks_ordered(si, off, T, order, states_out=states))
+        else:
+            ms = timed(lambda: pg.precog_encode_chunks(si, off, T, states_out=states))
         nb = scan_bytes_per_launch(T, shape.n_chunks, shape.D, shape.N, state_bytes=states.element_size())
         ct = T * shape.D
         row = {"ms_per_layer": ms, "tokens": T, "chunks": shape.n_chunks, "D": shape.D,
@@ -581,6 +589,8 @@ def measure_configs(pg, synth, torch, dev, hbm, alu_peak, cpu_chunks):
         else:
             row["layers"] = shape.n_layers
             row["tokens_per_s"] = T / (shape.n_layers * ms * 1e-3)   # through all 24 layers
+            row["order"] = "longest chunk first (precog_encode_chunks_ordered)"
+            row["ms_per_layer_unordered"] = ms_unordered
             out["ragged_encode"] = row
         r1 = int(off_np[cpu_chunks])
         samples[shape.name] = {k: inp[k][:r1].cpu().double().numpy() for k in ("x", "dt", "B")}

@@ -65,7 +65,8 @@ typedef enum precog_a_kind {
 
 /* Device status bits reported by precog_device_status(). */
 #define PRECOG_DEV_BAD_OFFSETS 0x1u  /* offsets not non-decreasing or beyond T_tot */
-#define PRECOG_DEV_BAD_INDEX 0x2u    /* a bank row index outside [-1, bank_entries) */
+#define PRECOG_DEV_BAD_INDEX 0x2u    /* a bank row index outside [-1, bank_entries), or a
+                                        chunk order entry outside [0, n_chunks) */
 #define PRECOG_DEV_TIMEOUT 0x4u      /* an mbarrier wait hit its iteration limit */
 #define PRECOG_DEV_BAD_A 0x8u        /* a_kind == PRECOG_A_POWER but A is not */
 
@@ -145,6 +146,26 @@ precog_status precog_encode_chunks(const precog_scan_inputs *in, const int64_t *
                                    int64_t n_chunks, int64_t T_tot, void *states_out,
                                    int32_t state_dtype, int32_t layer0, int32_t L_total,
                                    void *y_out, int32_t y_dtype, void *stream);
+
+/*
+ * precog_encode_chunks_ordered -- precog_encode_chunks with the order in which
+ * chunks are taken up (Sec. 4.2: chunks are independent, so any order gives the
+ * same states). With ragged chunks the last chunks to start decide when the
+ * launch ends; a caller that knows the lengths (it built d_offsets) can pass
+ * them longest first, so the short ones fill the tail.
+ *
+ *   d_order   device int64 [n_chunks]: work item i encodes chunk d_order[i],
+ *             and its state (and y rows) are written at that chunk's own index.
+ *             Meant to be a permutation of 0 .. n_chunks-1 (not verified: a
+ *             repeated chunk is written twice with the same result, a missing one
+ *             is not written). An entry outside [0, n_chunks) is skipped and
+ *             flags PRECOG_DEV_BAD_INDEX. NULL returns PRECOG_ERR_INVALID_ARG.
+ * Other arguments, layouts and errors as precog_encode_chunks.
+ */
+precog_status precog_encode_chunks_ordered(const precog_scan_inputs *in, const int64_t *d_offsets,
+                                           int64_t n_chunks, int64_t T_tot, const int64_t *d_order,
+                                           void *states_out, int32_t state_dtype, int32_t layer0,
+                                           int32_t L_total, void *y_out, int32_t y_dtype, void *stream);
 
 /*
  * precog_encode_trajectory -- the K-dial state trajectory of SMC (Sec. 5.2,

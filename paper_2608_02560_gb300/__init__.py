@@ -9,6 +9,7 @@ loudly: there is no CPU fallback.
 Functions carry the C names:
 
 * :func:`precog_encode_chunks`    -- offline indexing (Sec. 4.2)
+* :func:`precog_encode_chunks_ordered` -- the same, chunks taken up in a given order
 * :func:`precog_encode_trajectory` -- K-dial trajectory capture (Sec. 5.2)
 * :func:`precog_retrieve`         -- exact top-1 retrieval (Sec. 4.2)
 * :func:`precog_prefill_from_state` -- injection (Eq. 2) + query prefill
@@ -68,6 +69,9 @@ def load_library(path: str = LIB_PATH):
     lib.precog_encode_chunks.restype = i32
     lib.precog_encode_chunks.argtypes = [ctypes.POINTER(ScanInputs), vp, i64, i64, vp, i32, i32,
                                          i32, vp, i32, vp]
+    lib.precog_encode_chunks_ordered.restype = i32
+    lib.precog_encode_chunks_ordered.argtypes = [ctypes.POINTER(ScanInputs), vp, i64, i64, vp, vp, i32, i32,
+                                                 i32, vp, i32, vp]
     lib.precog_retrieve.restype = i32
     lib.precog_retrieve.argtypes = [vp, i32, i64, i32, vp, i32, vp, vp, vp, sz, vp]
     lib.precog_retrieve_keys.restype = i32
@@ -194,6 +198,27 @@ def precog_encode_chunks(inputs: ScanInputs, offsets, T_tot: int, states_out=Non
         ctypes.byref(inputs), _ptr(offsets), n_chunks, T_tot, _ptr(states_out),
         _dtype_code(states_out) if states_out is not None else PRECOG_F32, layer0, L_total,
         _ptr(y_out), _dtype_code(y_out) if y_out is not None else PRECOG_F32, _stream(stream)))
+
+
+def precog_encode_chunks_ordered(inputs: ScanInputs, offsets, T_tot: int, order, states_out=None,
+                                 layer0: int = 0, L_total: int | None = None, y_out=None, stream=None):
+    """:func:`precog_encode_chunks` taking chunks up in the order of ``order`` (device
+    int64 ``[n_chunks]``, a permutation, e.g. longest first); identical outputs."""
+    lib = load_library()
+    n_chunks = offsets.numel() - 1
+    if L_total is None:
+        L_total = inputs.n_layers
+    if order.numel() != n_chunks or order.dtype != _torch().int64:
+        raise ValueError("order must be int64 with one entry per chunk")
+    _check(lib.precog_encode_chunks_ordered(
+        ctypes.byref(inputs), _ptr(offsets), n_chunks, T_tot, _ptr(order), _ptr(states_out),
+        _dtype_code(states_out) if states_out is not None else PRECOG_F32, layer0, L_total,
+        _ptr(y_out), _dtype_code(y_out) if y_out is not None else PRECOG_F32, _stream(stream)))
+
+
+def _torch():
+    import torch
+    return torch
 
 
 def precog_encode_trajectory(inputs: ScanInputs, offsets, T_tot: int, stride: int, entry_offsets,

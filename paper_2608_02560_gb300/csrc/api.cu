@@ -135,12 +135,12 @@ cudaError_t ensure_smem(const void *kernel, int bytes) {
 
 }  // namespace precog
 
-extern "C" {
+namespace {
 
-precog_status precog_encode_chunks(const precog_scan_inputs *in, const int64_t *d_offsets,
-                                   int64_t n_chunks, int64_t T_tot, void *states_out,
-                                   int32_t state_dtype, int32_t layer0, int32_t L_total,
-                                   void *y_out, int32_t y_dtype, void *stream) {
+precog_status encode_chunks(const precog_scan_inputs *in, const int64_t *d_offsets, int64_t n_chunks,
+                            int64_t T_tot, void *states_out, int32_t state_dtype, int32_t layer0,
+                            int32_t L_total, void *y_out, int32_t y_dtype, const int64_t *d_order,
+                            void *stream) {
     if (T_tot < 0) return fail(PRECOG_ERR_INVALID_ARG, "T_tot must be >= 0");
     precog_status s = check_scan_inputs(in, T_tot, y_out != nullptr);
     if (s != PRECOG_OK) return s;
@@ -163,6 +163,7 @@ precog_status precog_encode_chunks(const precog_scan_inputs *in, const int64_t *
     if (n_chunks == 0) return ok();
     precog::ScanParams p = base_params(in, T_tot);
     p.offsets = d_offsets;
+    p.order = d_order;
     p.n_chunks = n_chunks;
     p.states = states_out;
     p.state_dtype = state_dtype;
@@ -175,6 +176,27 @@ precog_status precog_encode_chunks(const precog_scan_inputs *in, const int64_t *
                         : precog::launch_scan(p, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
     return ok();
+}
+
+}  // namespace
+
+extern "C" {
+
+precog_status precog_encode_chunks(const precog_scan_inputs *in, const int64_t *d_offsets,
+                                   int64_t n_chunks, int64_t T_tot, void *states_out,
+                                   int32_t state_dtype, int32_t layer0, int32_t L_total,
+                                   void *y_out, int32_t y_dtype, void *stream) {
+    return encode_chunks(in, d_offsets, n_chunks, T_tot, states_out, state_dtype, layer0, L_total, y_out,
+                         y_dtype, nullptr, stream);
+}
+
+precog_status precog_encode_chunks_ordered(const precog_scan_inputs *in, const int64_t *d_offsets,
+                                           int64_t n_chunks, int64_t T_tot, const int64_t *d_order,
+                                           void *states_out, int32_t state_dtype, int32_t layer0,
+                                           int32_t L_total, void *y_out, int32_t y_dtype, void *stream) {
+    if (d_order == nullptr) return fail(PRECOG_ERR_INVALID_ARG, "d_order is NULL");
+    return encode_chunks(in, d_offsets, n_chunks, T_tot, states_out, state_dtype, layer0, L_total, y_out,
+                         y_dtype, d_order, stream);
 }
 
 precog_status precog_prefill_from_state(const precog_scan_inputs *in, int32_t n_queries,

@@ -23,6 +23,9 @@ struct ScanParams {
     // else rows [offsets[c], offsets[c+1])
     const int64_t *offsets;
     int64_t n_chunks;
+    // processing order: work item i takes chunk order[i] (nullptr: chunk i); results are
+    // written at the chunk's own index, so any permutation gives the same outputs
+    const int64_t *order = nullptr;
     int32_t use_fixed;
     int32_t fixed_len;
     // initial state (prefill); bank == nullptr -> zero state

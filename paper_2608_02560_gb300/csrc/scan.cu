@@ -682,7 +682,11 @@ __global__ void __launch_bounds__(C::LB_THREADS, C::LB_BLOCKS)
     int64_t item = blockIdx.x;
     const int slice = static_cast<int>(item % slices);
     item /= slices;
-    const int64_t chunk = item % p.n_chunks;
+    const int64_t chunk = p.order ? p.order[item % p.n_chunks] : item % p.n_chunks;
+    if (chunk < 0 || chunk >= p.n_chunks) {  // an order entry outside the chunks: skipped
+        if (threadIdx.x == 0) atomicOr(&g_scan_status, PRECOG_DEV_BAD_INDEX);
+        return;
+    }
     const int layer = static_cast<int>(item / p.n_chunks);
     // this thread's rows of A first (16 floats each, 16-byte loads): their latency overlaps
     // the chunk's offsets below

@@ -356,7 +356,11 @@ __global__ void __launch_bounds__(block_channels<HAS_Y>())
     int64_t item = blockIdx.x;
     const int cb = static_cast<int>(item % cblocks);
     item /= cblocks;
-    const int64_t chunk = item % p.n_chunks;
+    const int64_t chunk = p.order ? p.order[item % p.n_chunks] : item % p.n_chunks;
+    if (chunk < 0 || chunk >= p.n_chunks) {  // an order entry outside the chunks: skipped
+        if (threadIdx.x == 0) atomicOr(&g_scan_complex_status, PRECOG_DEV_BAD_INDEX);
+        return;
+    }
     const int layer = static_cast<int>(item / p.n_chunks);
     const int D = p.D;
     const int d0 = cb * CB;

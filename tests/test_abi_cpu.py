@@ -103,6 +103,24 @@ def test_encode_rejects_bad_call_arguments(lib):
     assert _encode(lib, s, n_chunks=0) == 0                 # nothing to do: OK, no launch
 
 
+def test_ordered_encode_checks_its_arguments(lib):
+    """The ordered encode needs an order array and otherwise checks what the plain one
+    checks, before any launch."""
+    import paper_2608_02560_gb300 as pg
+    s = _inputs(pg)
+    f = lib.precog_encode_chunks_ordered
+    f.restype = ctypes.c_int32
+    f.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p,
+                  ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p,
+                  ctypes.c_int32, ctypes.c_void_p]
+    call = lambda order=FAKE, **kw: f(ctypes.byref(s), kw.get("offsets", FAKE), kw.get("n_chunks", 3), 64, order,
+                                      kw.get("states", FAKE), 0, 0, 1, None, 0, None)
+    assert call(order=None) == 1
+    assert call(offsets=None) == 1
+    assert call(states=FAKE + 8) == 1
+    assert call(n_chunks=0) == 0
+
+
 def test_prefill_rejects_bad_arguments(lib):
     import paper_2608_02560_gb300 as pg
     s = _inputs(pg)

@@ -416,3 +416,60 @@ def test_ragged_large_scale_encode_full_size(cuda_device):
     lens = np.diff(off)
     fixed = [int(np.argmax(lens)), int(np.argmin(lens)), 0, 4097, 8191]
     _sampled_check(cuda_device, synth.RAGGED, 5, _sample(8192, fixed, seed=5))
+
+
+@pytest.mark.parametrize("case", ["capture_bf16", "readout_f32", "few_chunks_readout", "complex"])
+def test_ordered_encode_matches_unordered(cuda_device, case):
+    """precog_encode_chunks_ordered: any processing order (random, longest first) gives
+    bit for bit the states (and y) of the plain call; an order entry outside the chunks
+    is skipped with PRECOG_DEV_BAD_INDEX and leaves that work item's chunk unwritten."""
+    import math
+    import torch
+    pg = _pg()
+    d = cuda_device
+    rng = np.random.default_rng(77)
+    few = case == "few_chunks_readout"
+    n = 5 if few else (200 if case == "readout_f32" else 40)
+    lens = rng.integers(0, 300, size=n)
+    lens[3] = 0
+    off_np = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    T = int(off_np[-1])
+    D, N = (256, 16) if case != "readout_f32" else (64, 16)
+    dtype = torch.bfloat16 if case in ("capture_bf16", "complex") else torch.float32
+    inp = synth.device_scan_inputs(T, D, N, 5, 0, d, dtype=dtype)
+    y_mode = case in ("readout_f32", "few_chunks_readout")
+    if case == "complex":
+        A = torch.complex(inp["A"], (math.pi * torch.arange(N, device=d, dtype=torch.float32)).expand(D, N))
+        si = pg.scan_inputs(inp["x"], inp["dt"], inp["B"], A.contiguous(), a_kind=pg.PRECOG_A_COMPLEX)
+        shape = (n, 1, D, N, 2)
+    else:
+        si = pg.scan_inputs(inp["x"], inp["dt"], inp["B"], inp["A"], inp["C"] if y_mode else None,
+                            a_kind=pg.PRECOG_A_POWER)
+        shape = (n, 1, D, N)
+    off = torch.from_numpy(off_np).to(d)
+
+    def run(order):
+        st = torch.full(shape, 7.0, dtype=torch.float32, device=d)
+        y = torch.full((1, T, D), 7.0, dtype=torch.float32, device=d) if y_mode else None
+        if order is None:
+            pg.precog_encode_chunks(si, off, T, states_out=st, y_out=y)
+        else:
+            pg.precog_encode_chunks_ordered(si, off, T, torch.from_numpy(order).to(d), states_out=st, y_out=y)
+        return st, y
+
+    ref_st, ref_y = run(None)
+    assert pg.precog_device_status()[0] == 0
+    for order in (rng.permutation(n).astype(np.int64), np.argsort(-lens, kind="stable").astype(np.int64)):
+        st, y = run(order)
+        assert pg.precog_device_status()[0] == 0
+        assert torch.equal(st, ref_st)
+        if y_mode:
+            assert torch.equal(y, ref_y)
+    bad = np.arange(n, dtype=np.int64)
+    bad[1] = n + 5                                   # chunk 1 is never taken up
+    st, _ = run(bad)
+    status, bits = pg.precog_device_status()
+    assert bits & pg.PRECOG_DEV_BAD_INDEX
+    assert bool((st[1] == 7.0).all())
+    keep = [c for c in range(n) if c != 1]
+    assert torch.equal(st[keep], ref_st[keep])
