@@ -139,13 +139,17 @@ def test_query_workload_full_index(cuda_device, Q):
 @pytest.mark.parametrize("dtype_name", ["float16", "bfloat16"])
 @pytest.mark.parametrize("M,Q,dim", [(1, 5, 64), (127, 9, 64), (128, 130, 96), (129, 256, 768),
                                      (4099, 300, 96), (20000, 17, 136), (3000, 2, 64), (70000, 4, 768),
-                                     (513, 127, 64), (513, 128, 64)])
+                                     (513, 127, 64), (513, 128, 64),
+                                     (1000, 200, 96), (39161, 300, 136), (77824, 129, 64)])
 def test_tensor_core_exact_integer_scores(cuda_device, dtype_name, M, Q, dim):
     """Every retrieval over a 16-bit index takes the tcgen05 path; these shapes stress
     its tiling. Small integer keys and queries make every score exact in fp32, so indices
     and scores must
     equal the oracle's bit for bit: ragged tiles (M), ragged and multi-pass query batches
-    (Q > 128, Q > 256), a K tail (dim not a multiple of 64), many exact ties."""
+    (Q > 128, Q > 256), a K tail (dim not a multiple of 64), many exact ties. A pass of
+    two query halves over an even number of CTAs runs as CTA pairs sharing the query
+    operand: 4 tiles on 4 CTAs (1000), 153 tiles on 152 CTAs so that one CTA of the first
+    pair runs a tile past the end (39161), a second half of one query (77824, 129)."""
     import torch
     dtype = getattr(torch, dtype_name)
     rng = np.random.default_rng(M * 31 + Q * 7 + dim)

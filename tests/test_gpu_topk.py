@@ -28,7 +28,8 @@ def _topk(index, queries, k):
 
 @pytest.mark.parametrize("dtype_name", ["float16", "bfloat16", "float32"])
 @pytest.mark.parametrize("M,Q,k,dim", [(1, 1, 3, 64), (5, 2, 8, 64), (1000, 3, 3, 96),
-                                       (4099, 9, 8, 64), (20000, 200, 5, 136), (300, 300, 2, 64)])
+                                       (4099, 9, 8, 64), (20000, 200, 5, 136), (300, 300, 2, 64),
+                                       (39161, 257, 3, 96), (77824, 129, 8, 64)])
 def test_topk_exact_integer_scores(cuda_device, dtype_name, M, Q, k, dim):
     """Small-integer keys: exact scores, many ties. Rows and scores must equal the
     oracle's stable ranking bit for bit, on the CUDA-core path (fp32 keys) and the
