@@ -147,9 +147,9 @@ def test_tensor_core_exact_integer_scores(cuda_device, dtype_name, M, Q, dim):
     and scores must
     equal the oracle's bit for bit: ragged tiles (M), ragged and multi-pass query batches
     (Q > 128, Q > 256), a K tail (dim not a multiple of 64), many exact ties. A pass of
-    two query halves over an even number of CTAs runs as CTA pairs sharing the query
-    operand: 4 tiles on 4 CTAs (1000), 153 tiles on 152 CTAs so that one CTA of the first
-    pair runs a tile past the end (39161), a second half of one query (77824, 129)."""
+    more than 128 queries over an even grid runs on SM pairs (one M = 256 MMA per pair):
+    4 tiles on 2 pairs (1000), 153 tiles on 76 pairs so that the first pair takes a third
+    tile (39161), a second half of one query (77824, 129)."""
     import torch
     dtype = getattr(torch, dtype_name)
     rng = np.random.default_rng(M * 31 + Q * 7 + dim)
