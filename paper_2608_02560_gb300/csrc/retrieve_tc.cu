@@ -43,10 +43,6 @@ constexpr int kStages = 3;
 constexpr int kTopkStride = 8;    // keys per (CTA, query) in the top-k workspace
 constexpr int kThreads = 320;     // 2 control warps + 8 epilogue warps
 constexpr uint32_t kTmemCols = 512;
-#ifndef PRECOG_TC_PAIRS
-#define PRECOG_TC_PAIRS 1
-#endif
-constexpr bool kUsePairs = PRECOG_TC_PAIRS != 0;
 constexpr uint32_t kABytes = kBM * kBK * 2;   // one query half per stage
 constexpr uint32_t kBBytes = kBN * kBK * 2;
 
@@ -593,7 +589,7 @@ cudaError_t launch_tc(const RetrieveParams &p, int grid, cudaStream_t stream, ui
     cudaError_t e = ensure_smem(reinterpret_cast<const void *>(retrieve_tc_kernel<LIST>), smem);
     if (e != cudaSuccess) return e;
     // Passes of more than 128 queries run on SM pairs when the grid splits into pairs.
-    const bool pairs = kUsePairs && grid % 2 == 0 && p.n_queries > kBM;
+    const bool pairs = grid % 2 == 0 && p.n_queries > kBM;
     CUtensorMap tk_pair;
     const int smem_pair = static_cast<int>(sizeof(PairSmem<LIST>) + 1024);
     if (pairs) {
