@@ -55,7 +55,7 @@ __device__ uint32_t g_scan_status;
 #define PRECOG_DIRECT_STAGES 2
 #endif
 #ifndef PRECOG_DIRECT_MINB
-#define PRECOG_DIRECT_MINB 6
+#define PRECOG_DIRECT_MINB 5
 #endif
 #ifndef PRECOG_RESCALED_GROUP
 #define PRECOG_RESCALED_GROUP 4
