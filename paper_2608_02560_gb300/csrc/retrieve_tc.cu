@@ -340,14 +340,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 // ---------------------------------------------------------------------------------------
 // SM pairs for a pass of more than 128 queries (cta_group::2).
 //
-// With two 128-query halves on one SM, every k-block has the MMAs read 96 KB of operands
-// from shared memory (the key tile once per half) while the copies write another 64 KB
-// into it, and the two accumulators fill tensor memory, so each tile's MMAs also wait for
-// the previous tile's epilogue. A cluster of two CTAs runs one M = 256 MMA instead: CTA r
-// stages only its own 128 queries (rows r*128.. of A) and 128 of the tile's 256 keys
-// (rows r*128.. of B), 32 KB per k-block, and holds the 128 x 256 scores of its own
-// queries in its own tensor memory. 256 columns per tile leave room for two buffers, so
-// the epilogue overlaps the next tile's MMAs again.
+// With two 128-query halves on one SM the two accumulators fill all 512 TMEM columns, so
+// each tile's MMAs wait for the previous tile's epilogue. A cluster of two CTAs runs one
+// M = 256 MMA instead: CTA r stages only its own 128 queries (rows r*128.. of A) and 128
+// of the tile's 256 keys (rows r*128.. of B), 32 KB per k-block, and holds the 128 x 256
+// scores of its own queries in its own tensor memory. 256 columns per tile leave room for
+// two buffers, so the epilogue overlaps the next tile's MMAs again. (Shared-memory traffic
+// per multiply-add is unchanged: each SM's B half is read by both tensor cores.)
 //
 // Roles (both CTAs unless noted): warp 0 TMA producer of this CTA's query and key rows,
 // counted on the even CTA's full barrier; warp 1 TMEM allocation (collective over the
