@@ -862,9 +862,10 @@ def main():
     if not args.no_e2e:
         # one pinned host copy per resident input set, so that layer l streams set l mod S's
         # inputs from the host and the e2e bank equals the timed region's
-        # (when the host cannot pin that much, the sets share one host copy)
+        # (when the host cannot pin that much for every rank on it, the sets share one copy)
         set_bytes = sum(sets[0][k].numel() * sets[0][k].element_size() for k in ("x", "dt", "B"))
-        HS = S if host_available_bytes() > 2 * S * set_bytes else 1
+        local_ranks = int(os.environ.get("LOCAL_WORLD_SIZE", "1"))
+        HS = S if host_available_bytes() > 2 * S * set_bytes * local_ranks else 1
         host = [{k: torch.empty(sets[s_][k].shape, dtype=sets[s_][k].dtype, pin_memory=True)
                  for k in ("x", "dt", "B")} for s_ in range(HS)]
         for s_ in range(HS):
