@@ -141,6 +141,43 @@ def test_multi_layer_call_and_layer_offset(cuda_device):
             assert rel_err(got[c, 2 + l], ref[c]) < TOL_F32
 
 
+def test_concurrent_calls_on_two_streams_write_disjoint_layers(cuda_device):
+    """Encode calls that write disjoint layers of one bank may run at the same time on two
+    streams (the benchmark's step alternates its calls that way): the bank equals the one
+    written by the same calls one after the other, bit for bit, and every entry is written."""
+    import torch
+    pg = _pg()
+    d = cuda_device
+    n_chunks, clen, D, N = 304, 1000, 256, 16
+    T = n_chunks * clen
+    sets = [synth.device_scan_inputs(T, D, N, 70, l, d, with_C=False) for l in range(4)]
+    off = torch.from_numpy(synth.fixed_offsets(n_chunks, clen)).to(d)
+
+    def call_inputs(first):
+        st = lambda k: torch.stack([sets[first + i][k] for i in range(2)]).contiguous()
+        return pg.scan_inputs(st("x"), st("dt"), st("B"), st("A"), a_kind=pg.PRECOG_A_POWER)
+
+    calls = [call_inputs(0), call_inputs(2)]
+    seq = torch.full((n_chunks, 4, D, N), float("nan"), dtype=torch.bfloat16, device=d)
+    for c in range(2):
+        pg.precog_encode_chunks(calls[c], off, T, states_out=seq, layer0=2 * c, L_total=4)
+    torch.cuda.synchronize()
+    conc = torch.full_like(seq, float("nan"))
+    streams = [torch.cuda.Stream(device=d), torch.cuda.Stream(device=d)]
+    start = torch.cuda.Event()
+    start.record()
+    for c in range(2):
+        streams[c].wait_event(start)
+        pg.precog_encode_chunks(calls[c], off, T, states_out=conc, layer0=2 * c, L_total=4,
+                                stream=streams[c])
+    for s_ in streams:
+        torch.cuda.current_stream(d).wait_stream(s_)
+    torch.cuda.synchronize()
+    assert pg.precog_device_status()[0] == 0
+    assert bool(torch.isfinite(seq.float()).all())
+    assert torch.equal(conc, seq)
+
+
 @pytest.mark.parametrize("D,y_mode,dtype_name", [(512, False, "float32"), (1024, False, "float32"),
                                                  (768, False, "float32"), (4096, False, "float32"),
                                                  (1024, True, "float32"), (768, True, "float32"),
